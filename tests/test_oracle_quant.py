@@ -1,0 +1,208 @@
+"""Pins of the oracle's levels, fitted scales, storage layout and bit accounting (Sec. 3,
+"Levels and storage"), and of the log-uniform decay-gate quantiser (Sec. 3, "Decay-gate
+quantization")."""
+import os
+
+import numpy as np
+import pytest
+
+GOLD = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _f16(x):
+    return int(np.array(np.float16(np.clip(np.float32(x), -65504, 65504))).view(np.uint16))
+
+
+def test_fp16_scale_rounding_matches_ieee(orc):
+    """The 1-bit scale is FP16(mean |x|): compare with numpy's IEEE binary16 (RNE)."""
+    rng = np.random.default_rng(0)
+    vals = np.concatenate([np.exp(rng.uniform(-20, 12, 2000)), [6.1e-5, 5.9e-8, 2.9e-8, 65504,
+                                                                 65519, 65520, 1e6, 1.0]])
+    for v in vals.astype(np.float32):
+        _, scale, _ = orc.quant_group(np.full(8, v, np.float32), 1)
+        assert scale == _f16(v), v
+
+
+def test_fit_grid_and_scale_formula(orc):
+    """16 factors evenly spaced on [1/4, 1]; Delta = FP16(f R (1/n)); with fidx forced the
+    stored scale follows the formula exactly."""
+    rng = np.random.default_rng(1)
+    x = (rng.standard_normal(64) * 3).astype(np.float32)
+    R = np.float32(np.max(np.abs(x)))
+    for b in (2, 3, 4, 8, 12, 16):
+        n = 2 ** (b - 1) - 1
+        for k in range(16):
+            f = np.float32((5 + k) / 20)
+            _, scale, fidx = orc.quant_group(x, b, refit=False, fidx_in=k)
+            assert fidx == k
+            assert scale == _f16(np.float32(f * R) * np.float32(np.float32(1) / np.float32(n)))
+    assert np.float32((5 + 0) / 20) == np.float32(0.25) and np.float32((5 + 15) / 20) == 1.0
+
+
+@pytest.mark.parametrize("b", [2, 3, 4, 5, 8, 11, 16])
+def test_chosen_factor_minimises_squared_error(orc, b):
+    """The fitted f has the smallest squared error of the 16 candidates: every candidate is
+    re-quantised on its own (fidx forced), dequantised and scored in FP64 here."""
+    rng = np.random.default_rng(b)
+    for trial in range(40):
+        g = int(rng.choice([32, 64, 128]))
+        x = (rng.standard_t(3, g) * np.exp(rng.normal(0, 2))).astype(np.float32)
+        codes, scale, fidx = orc.quant_group(x, b)
+        sse = []
+        for k in range(16):
+            ck, sk, _ = orc.quant_group(x, b, refit=False, fidx_in=k)
+            xh = orc.dequant_group(ck, b, sk).astype(np.float64)
+            sse.append(float(np.sum((x.astype(np.float64) - xh) ** 2)))
+        sse = np.array(sse)
+        # FP32 accumulation in the oracle may reorder candidates within its rounding error
+        assert sse[fidx] <= sse.min() * (1 + 1e-5) + 1e-30
+        xh = orc.dequant_group(codes, b, scale)
+        assert np.all(codes <= 2 ** b - 2)
+        n = 2 ** (b - 1) - 1
+        D = np.float16(np.array(scale, np.uint16).view(np.float16)).astype(np.float32)
+        assert np.array_equal(xh, ((codes.astype(np.int64) - n).astype(np.float32) * D))
+
+
+def test_two_bit_levels_and_exact_range_round_trip(orc):
+    """b = 2: levels {-Delta, 0, Delta}.  With f = 1 and an FP16-exact R/n, +-R round-trips."""
+    rng = np.random.default_rng(2)
+    x = rng.standard_normal(128).astype(np.float32)
+    codes, scale, _ = orc.quant_group(x, 2)
+    D = float(np.array(scale, np.uint16).view(np.float16))
+    assert set(np.unique(codes)) <= {0, 1, 2}
+    assert set(np.unique(orc.dequant_group(codes, 2, scale))) <= {-D, 0.0, D}
+    for b in (2, 4, 7, 10):
+        n = 2 ** (b - 1) - 1
+        R = np.float32(n * 0.375)                      # R / n = 0.375 is exact in FP16
+        x = rng.uniform(-R, R, 96).astype(np.float32)
+        x[3], x[50] = R, -R
+        codes, scale, _ = orc.quant_group(x, b, refit=False, fidx_in=15)
+        xh = orc.dequant_group(codes, b, scale)
+        assert xh[3] == R and xh[50] == -R
+        assert np.all(np.abs(xh - x) <= 0.375 / 2 + 1e-7)
+
+
+def test_one_bit_is_sign_times_mean(orc):
+    x = np.array([0.5, -1.5, 0.0, -0.0, 2.0, -3.0, 1.0, 0.25], np.float32)
+    codes, scale, _ = orc.quant_group(x, 1)
+    assert list(codes) == [0, 1, 0, 0, 0, 1, 0, 0]
+    m = np.float16(np.float32(np.sum(np.abs(x))) / np.float32(8))
+    assert scale == int(np.array(m).view(np.uint16))
+    assert np.array_equal(orc.dequant_group(codes, 1, scale),
+                          np.where(codes == 1, -np.float32(m), np.float32(m)))
+
+
+def test_zero_group_and_zero_width(orc):
+    codes, scale, fidx = orc.quant_group(np.zeros(32, np.float32), 5)
+    assert scale == 0 and np.all(codes == 15) and fidx == 15
+    assert np.all(orc.dequant_group(codes, 5, scale) == 0)
+    assert np.all(orc.dequant_group(np.zeros(32, np.uint16), 0, 0) == 0)
+
+
+def test_pack_layout_golden(orc):
+    for line in open(os.path.join(GOLD, "pack_layout.txt")):
+        line = line.strip()
+        if not line or line.startswith("#"):
+            continue
+        lhs, rhs = line.split("->")
+        b, *codes = [int(t) for t in lhs.split()]
+        want = bytes(int(t, 16) for t in rhs.split())
+        got = orc.pack_codes(np.array(codes, np.uint16), b).tobytes()
+        assert got == want, (b, codes, got.hex(), want.hex())
+
+
+@pytest.mark.parametrize("b", range(1, 17))
+def test_pack_unpack_identity(orc, b):
+    rng = np.random.default_rng(b)
+    for g in (8, 32, 64, 128):
+        codes = rng.integers(0, 2 ** b, g).astype(np.uint16)
+        packed = orc.pack_codes(codes, b)
+        assert packed.size == b * g // 8
+        assert np.array_equal(orc.unpack_codes(packed, g, b), codes)
+
+
+def test_state_pack_unpack_round_trip_error(orc):
+    """Whole-state pack/unpack: dequantised error per element <= Delta/2 inside the range and
+    widths/offsets follow the prefix-sum layout."""
+    import synth
+    w = synth.scaled(synth.WORKLOADS["kda_decode"], B=2, H=3, dk=32, dv=32)
+    cfg = orc.Cfg.from_workload(w)
+    rng = np.random.default_rng(3)
+    pool = np.array([0, 8, 1, 7, 2, 6, 3, 5, 4] * 10 + [4] * 6)     # 96 rows, mean exactly 4
+    assert pool.size == cfg.units and pool.sum() == cfg.units * 4
+    wb = np.stack([rng.permutation(pool) for _ in range(cfg.B)])
+    widths = wb.astype(np.uint8).ravel()
+    row_bytes = wb.reshape(cfg.B, cfg.H, cfg.dk) * cfg.dv // 8
+    head_off = np.concatenate([np.zeros((cfg.B, 1), int), np.cumsum(row_bytes.sum(2), 1)[:, :-1]],
+                              1).astype(np.uint32).ravel()
+    S = synth.random_state(w, 1)
+    payload, scales, fidx, rng_out = orc.pack(cfg, S, widths, head_off)
+    X = orc.unpack(cfg, payload, scales, widths, head_off)
+    R = np.max(np.abs(S), axis=3).ravel()
+    assert np.array_equal(rng_out, R)
+    D = np.array(scales, np.uint16).view(np.float16).astype(np.float32)
+    Dr = D.reshape(cfg.B, cfg.H, cfg.dk, 1)
+    wr = widths.reshape(cfg.B, cfg.H, cfg.dk, 1)
+    n = (2.0 ** (wr - 1) - 1)
+    inside = (np.abs(S) <= (n + 0.5) * Dr) & (wr >= 2)
+    assert np.all(np.abs(X - S)[inside] <= Dr.repeat(cfg.dv, 3)[inside] / 2 * (1 + 1e-6))
+    one = np.broadcast_to(wr == 1, S.shape)
+    assert np.all(np.abs(np.abs(X[one]) - np.broadcast_to(Dr, S.shape)[one]) == 0)
+
+
+def test_bits_accounting_matches_tables(orc):
+    """Table 2(a) / Table 3 totals from the metadata rule of Sec. 3."""
+    for line in open(os.path.join(GOLD, "bits_accounting.txt")):
+        line = line.strip()
+        if not line or line.startswith("#"):
+            continue
+        unit, bbar, bmin, bmax, dk, dv, total, src = line.split()
+        bbar, dk, dv = int(bbar), int(dk), int(dv)
+        if unit in ("int_row", "int_block"):
+            bmin = bmax = bbar
+            unit_kind = 0 if unit == "int_row" else 1
+        else:
+            bmin, bmax = int(bmin), int(bmax)
+            unit_kind = 0 if unit == "row" else 1
+        cfg = orc.Cfg(B=1, H=1, dk=dk, dv=dv, unit_kind=unit_kind, bbar_num=bbar, bmin=bmin,
+                      bmax=bmax)
+        got = orc.bits_per_element(cfg)
+        nd = len(total.split(".")[1]) if "." in total else 0
+        assert round(got, nd) == float(total), (src, got)
+
+
+# ------------------------------- log-uniform decay quantiser -------------------------------
+@pytest.mark.parametrize("g", [1, 2, 3, 4])
+def test_log_decay_levels_thresholds_codes(orc, g):
+    rng = np.random.default_rng(g)
+    nchan, count = 12, 500
+    s = np.log1p(np.exp(rng.normal(-2, 1, (count, nchan)))).astype(np.float32)
+    codes, lut, thr = orc.quant_decay(s, nchan, g)
+    L = 2 ** g
+    assert lut.shape == (nchan, L) and codes.max() <= L - 1
+    assert np.array_equal(lut[:, 0], s.min(0)) and np.array_equal(lut[:, -1], s.max(0))
+    # uniform in log s
+    ll = np.log(lut.astype(np.float64))
+    assert np.allclose(np.diff(ll, axis=1), (ll[:, -1:] - ll[:, :1]) / (L - 1), rtol=1e-5)
+    # thresholds are geometric means of neighbouring levels
+    gm = np.sqrt(lut[:, :-1].astype(np.float64) * lut[:, 1:])
+    assert np.allclose(thr, gm, rtol=1e-6)
+    # codes: monotone in s, each level maps to its own code, nearest level in log domain
+    for ch in range(nchan):
+        order = np.argsort(s[:, ch], kind="stable")
+        assert np.all(np.diff(codes[order, ch].astype(int)) >= 0)
+        lv = orc.quant_decay(np.concatenate([s[:, ch:ch + 1], lut[ch][:, None]]), 1, g)[0][-L:, 0]
+        assert list(lv) == list(range(L))
+        dist = np.abs(np.log(s[:, ch:ch + 1].astype(np.float64)) - ll[ch][None, :])
+        nearest = np.argmin(dist, axis=1)
+        ok = (codes[:, ch] == nearest) | (np.abs(np.sort(dist, 1)[:, 0] - np.sort(dist, 1)[:, 1])
+                                          < 1e-6)
+        assert np.all(ok)
+
+
+def test_log_decay_degenerate_and_invalid(orc):
+    s = np.full((10, 3), 0.2, np.float32)
+    codes, lut, _ = orc.quant_decay(s, 3, 2)
+    assert np.all(lut == np.float32(0.2)) and np.all(codes == 3)
+    with pytest.raises(ValueError):
+        orc.quant_decay(np.zeros((4, 2), np.float32), 2, 2)
