@@ -1,0 +1,200 @@
+/*
+ * qstate.h -- C ABI of libqstate: recurrent states of gated linear recurrences stored at low,
+ * variable bit width, after "Low-Bit Recurrent States in Hybrid Language Models"
+ * (Chen & He, 2026).
+ *
+ * One head's state S (dk x dv, rows = key channels, columns = value channels) follows Eq. (1):
+ *     S_t = (I - k_t a_t^T) D_t S_{t-1} + k_t (w_t o v_t)^T,   o_t = S_t^T q_t,
+ *     D_t = diag(e^{-s_t}),
+ * with a = beta k, w = beta 1 for KDA and Gated DeltaNet, and a = 0, w = 1 for Mamba-2.
+ * Every C tokens (Sec. 2, "Accumulated readout error") the state is written back: quantised
+ * with per-unit widths and FP16 range scales (Sec. 3, "Levels and storage") and dequantised
+ * before reuse; readouts are taken before quantising.  Widths come from the allocation of
+ * Sec. 3 (Eq. 3 weights, Eq. 4 and integer rounding to the layer budget).
+ *
+ * Conventions for every call:
+ *  - Pointers marked "device" are CUDA device pointers owned by the caller; the library never
+ *    allocates, frees or retains them.  Host structs are read during the call only.
+ *  - `stream` is a cudaStream_t (NULL = legacy default stream).  Work is enqueued
+ *    asynchronously on it; the call returns once it is enqueued.
+ *  - Arguments are validated on the host before anything is launched.  The return value is
+ *    QSTATE_OK or an error code; qstate_last_error() (per host thread) describes the last
+ *    failure.  No C++ exception crosses this interface.
+ *  - Kernels that find an inconsistent device-side layout (a width above 16, offsets running
+ *    past a region, a non-positive decay rate) skip the offending work and set a device status
+ *    word; qstate_check() synchronises the stream and reports it.
+ *  - All tensors are dense, C-contiguous, float32 unless stated.  Token-major inputs have
+ *    shape (B, T, H, d) with T the token extent given in qstate_inputs.
+ */
+#ifndef QSTATE_H
+#define QSTATE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ---------------------------------------------------------------------- */
+#define QSTATE_OK 0
+#define QSTATE_EINVAL 1  /* invalid argument or configuration                                */
+#define QSTATE_EBUDGET 2 /* N*bmin > N*bbar or N*bbar > N*bmax: the layer budget is unmeetable */
+#define QSTATE_ECUDA 3   /* a CUDA runtime call failed (message in qstate_last_error)          */
+#define QSTATE_EDEVICE 4 /* a kernel reported an inconsistent device-side layout or input      */
+
+/* ---- configuration enums ---------------------------------------------------------------- */
+#define QSTATE_DECAY_ROW 0   /* one rate per key row (KDA, Sec. 1)                            */
+#define QSTATE_DECAY_HEAD 1  /* one rate per head (Gated DeltaNet, Mamba-2)                   */
+#define QSTATE_ERASE_DELTA 0 /* a = beta k, w = beta 1 (Eq. 1, KDA / Gated DeltaNet)          */
+#define QSTATE_ERASE_NONE 1  /* a = 0, w = 1 (Eq. 1, Mamba-2)                                  */
+#define QSTATE_UNIT_ROW 0    /* width + FP16 scale per row (Sec. 3, "Allocation units")       */
+#define QSTATE_UNIT_HEAD 1   /* width per head, FP16 scale per 32 key rows x value column     */
+#define QSTATE_WEIGHT_OURS 0 /* c_i = Gamma_hat_i Rtilde_i^2 (Eq. 3)                           */
+
+/* Method configuration.  Sizes: dk in {64, 128}, dv in {64, 128}; dk a multiple of 32 for the
+ * head unit; the budget H*dk*dv*bbar must be a whole number of bytes per batch element. */
+typedef struct qstate_cfg {
+    int32_t B, H, dk, dv;
+    int32_t decay_kind;          /* QSTATE_DECAY_*                                           */
+    int32_t erase_kind;          /* QSTATE_ERASE_*                                           */
+    int32_t unit_kind;           /* QSTATE_UNIT_*; the head unit requires per-head decay     */
+    int32_t group_heads;         /* heads per output-normalisation group u(i), row unit (Sec. 2
+                                    "Range normalization"); must divide H                    */
+    int32_t bbar_num, bbar_den;  /* mean payload bits per element bbar = num/den (Eq. 4)      */
+    int32_t bmin, bmax;          /* width limits, 0 <= bmin <= bbar <= bmax <= 16 (Sec. 3)    */
+    int32_t C;                   /* write-back period in tokens (Sec. 2), >= 1               */
+    int32_t fit_every;           /* 1: fit the range factor f at every write-back (Sec. 3);
+                                    K > 1: head h refits when (write-back + h) % K == 0 and
+                                    otherwise reuses its stored factor                       */
+    float ema_span;              /* EMA span in tokens (Sec. 3: 64)                           */
+    int32_t gate_bits;           /* 0: FP32 decay rates; g in 1..8: log-quantised rates       */
+    int32_t weight_kind;         /* QSTATE_WEIGHT_OURS                                       */
+} qstate_cfg;
+
+/* One packed state (device pointers).  Layout (Sec. 3, "Levels and storage"; bit order is
+ * this library's reading):
+ *  payload  B regions of qstate_region_bytes() bytes.  In region b, head h starts at byte
+ *           head_off[b*H + h]; its rows follow in order, row i taking width_i*dv/8 bytes; row
+ *           element j's code occupies row bits [j*w, j*w + w), bit m of a row being bit m%8
+ *           of byte m/8.  Codes: w >= 2 -> offset binary q + n, n = 2^(w-1) - 1; w = 1 ->
+ *           sign bit (1 = negative); w = 0 -> nothing stored.
+ *  scales   FP16 bit patterns, one per scale group: (B, H, dk) for the row unit, (B, H, dk/32,
+ *           dv) for the head unit.  w >= 2: step Delta; w = 1: mean |x|.
+ *  widths   uint8, (B, H, dk) for the row unit, (B, H) for the head unit.
+ *  head_off uint32, (B, H), byte offsets inside the batch element's region.
+ *  fidx     uint8, one per scale group: index k of the fitted factor f_k = (5 + k)/20. */
+typedef struct qstate_buf {
+    uint8_t* payload;
+    uint16_t* scales;
+    uint8_t* widths;
+    uint32_t* head_off;
+    uint8_t* fidx;
+} qstate_buf;
+
+/* Per-unit statistics (device, float32, B*units each; units = H*dk row unit, H head unit):
+ *  ema_s  EMA of 1 - e^{-2 s} (the complement of the EMA of the squared decay factor, Sec. 3)
+ *  ema_r  EMA of beta (2 - beta) k_i^2 (row unit) or of beta (2 - beta) |k|^2 / dk (head unit)
+ *  range  row absolute maximum R_i of the state at the last write-back (row unit only). */
+typedef struct qstate_stats {
+    float* ema_s;
+    float* ema_r;
+    float* range;
+} qstate_stats;
+
+/* Token inputs (device).  q, k: (B, T, H, dk); v: (B, T, H, dv); s: (B, T, H, dk) for per-row
+ * decay or (B, T, H) for per-head decay, all rates > 0; beta: (B, T, H), ignored without
+ * erasure.  With log-quantised rates pass s = NULL, s_code (uint8, same shape as s) and
+ * s_lut (channels x 2^gate_bits levels, channels = H*dk or H) from qstate_quant_decay. */
+typedef struct qstate_inputs {
+    const float* q;
+    const float* k;
+    const float* v;
+    const float* s;
+    const uint8_t* s_code;
+    const float* s_lut;
+    const float* beta;
+    int32_t T;
+} qstate_inputs;
+
+/* ---- sizes and accounting (host only) ---------------------------------------------------- */
+/* QSTATE_OK if the configuration is supported; otherwise an error code + message. */
+int qstate_validate(const qstate_cfg* cfg);
+/* Payload bytes of one batch element: H*dk*dv*bbar/8 (0 if invalid). */
+size_t qstate_region_bytes(const qstate_cfg* cfg);
+/* Allocation units per batch element (H*dk or H) and scale groups per batch element. */
+size_t qstate_units(const qstate_cfg* cfg);
+size_t qstate_scale_groups(const qstate_cfg* cfg);
+/* Total stored bits per state element (Sec. 3): bbar + (16 + width bits)/dv for the row unit,
+ * bbar + 16/32 + width bits/(dk dv) for the head unit; width bits = ceil(log2(bmax-bmin+1)). */
+double qstate_bits_per_element(const qstate_cfg* cfg);
+
+/* ---- calls -------------------------------------------------------------------------------- */
+/* Initial state (Sec. 3 protocol): widths of the allocation with equal weights (uniform bbar
+ * when it is an integer), matching head offsets, and the zero state packed into `a`
+ * (scales 0, factor index 15).  `b` receives the same widths and offsets. */
+int qstate_init(const qstate_cfg* cfg, qstate_buf* a, qstate_buf* b, void* stream);
+
+/* Sec. 3, Eq. (3) and Eq. (4) + "round, clip to [b_min, b_max], and adjust widths to meet the
+ * layer budget": per batch element, weights c_i = Gamma_hat_i Rtilde_i^2 from `stats`
+ * (Gamma_hat = (1 - ema_s)/(expm1(ema_r) + ema_s), Rtilde_i^2 = R_i^2 / mean over the group of
+ * R^2, 1 for the head unit) and integer widths summing exactly to units*bbar: the widths that
+ * minimise sum_i c_i 4^{-w_i} under the limits, ties going to lower unit indices.  Writes
+ * widths_out (B*units) and head_off_out (B*H).  Bit-reproducible. */
+int qstate_alloc_bits(const qstate_cfg* cfg, const qstate_stats* stats, uint8_t* widths_out,
+                      uint32_t* head_off_out, void* stream);
+
+/* Sec. 3, "Levels and storage": quantise the dense state S (device, (B, H, dk, dv)) with the
+ * widths and offsets already in `out` (fitting f for every scale group) and write payload,
+ * scales and fidx of `out`; range_out (device, B*units, may be NULL) receives the row absmax. */
+int qstate_pack(const qstate_cfg* cfg, const float* S, qstate_buf* out, float* range_out,
+                void* stream);
+
+/* Inverse of qstate_pack: dequantise `in` into S_out (device, (B, H, dk, dv)). */
+int qstate_unpack(const qstate_cfg* cfg, const qstate_buf* in, float* S_out, void* stream);
+
+/* Sec. 3, "Decay-gate quantization": per channel (h, i) (or per head), levels uniform in
+ * log s between the smallest and largest rate over all (b, t): l_k = exp(lo + k (hi-lo)/(L-1)),
+ * L = 2^gate_bits, thresholds at the geometric means of neighbours, code = number of
+ * thresholds <= s.  s: device (B, T, H, dk) or (B, T, H); code_out: uint8, same shape;
+ * lut_out: channels x L levels; thr_out: channels x (L - 1) thresholds.  EDEVICE (from
+ * qstate_check) if a rate is not a positive finite number. */
+int qstate_quant_decay(const qstate_cfg* cfg, const float* s, int32_t T, uint8_t* code_out,
+                       float* lut_out, float* thr_out, void* stream);
+
+/* One write-back interval: tokens [t_begin, t_end) (at most C of them) of every head, from the
+ * state packed in `in` to `out` (whose widths and offsets must already hold the target
+ * allocation).  Unpack + dequantise, decay, delta update and readout o_t (device,
+ * (B, T, H, dv), read before quantising), EMA statistics, range fit, requantise + repack;
+ * then the allocation for the next write-back from the new statistics is written into
+ * in->widths / in->head_off (in's payload is dead by then), so the next interval runs with
+ * the roles of `in` and `out` swapped.  t = 0 initialises the EMAs.  w_index numbers this
+ * write-back (for fit_every). */
+int qstate_step(const qstate_cfg* cfg, qstate_buf* in, qstate_buf* out,
+                const qstate_inputs* x, int32_t t_begin, int32_t t_end, int32_t w_index,
+                float* o, qstate_stats* stats, void* stream);
+
+/* Tokens [t_begin, t_end) in write-back intervals of C tokens (the last one may be shorter),
+ * ping-ponging between `ping` (holding the state at t_begin, with pong's widths set as the
+ * first target) and `pong`.  *final_in_pong is set to 1 if the final state is in `pong`.
+ * Equal to the sequence of qstate_step calls, bit for bit.  w_index0 numbers the first
+ * write-back. */
+int qstate_scan(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong,
+                const qstate_inputs* x, int32_t t_begin, int32_t t_end, int32_t w_index0,
+                float* o, qstate_stats* stats, int32_t* final_in_pong, void* stream);
+
+/* Unquantised reference path: Eq. (1) on a dense FP32 state S (device, (B, H, dk, dv), in/out)
+ * for tokens [t_begin, t_end), the state round-tripping through memory every C tokens. */
+int qstate_scan_fp32(const qstate_cfg* cfg, float* S, const qstate_inputs* x, int32_t t_begin,
+                     int32_t t_end, float* o, void* stream);
+
+/* Synchronise `stream`, read and clear the device status word: QSTATE_OK or QSTATE_EDEVICE. */
+int qstate_check(void* stream);
+
+/* Message for the last failure on this host thread ("" if none).  Valid until the next call. */
+const char* qstate_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* QSTATE_H */

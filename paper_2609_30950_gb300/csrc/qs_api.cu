@@ -1,0 +1,413 @@
+// qs_api.cu -- the C ABI of libqstate (declared in include/qstate.h): host-side validation,
+// error reporting and kernel dispatch.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include "qs_internal.h"
+
+namespace qs {
+cudaError_t launch_step_128x128(const qstate_cfg&, int, int, const StepParams&, cudaStream_t);
+cudaError_t launch_step_128x64(const qstate_cfg&, int, int, const StepParams&, cudaStream_t);
+cudaError_t launch_step_64x64(const qstate_cfg&, int, int, const StepParams&, cudaStream_t);
+}  // namespace qs
+
+using namespace qs;
+
+// Device status word (QS_DEV_* bits).  Kernels receive its address; see status_word().
+static __device__ int qs_status_word;
+
+namespace {
+
+thread_local char g_err[512] = "";
+
+int fail(int code, const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof(g_err), fmt, ap);
+    va_end(ap);
+    return code;
+}
+
+int cuda_fail(cudaError_t e, const char* what) {
+    return fail(QSTATE_ECUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+constexpr int kMaxDevices = 64;
+std::mutex g_mu;
+int* g_status_addr[kMaxDevices] = {};
+
+// Address of the status word on the current device, looked up once per device.
+int* status_word(cudaError_t* err) {
+    int dev = 0;
+    *err = cudaGetDevice(&dev);
+    if (*err != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+    std::lock_guard<std::mutex> lock(g_mu);
+    if (!g_status_addr[dev]) {
+        void* p = nullptr;
+        *err = cudaGetSymbolAddress(&p, qs_status_word);
+        if (*err != cudaSuccess) return nullptr;
+        g_status_addr[dev] = static_cast<int*>(p);
+    }
+    return g_status_addr[dev];
+}
+
+long long units_of(const qstate_cfg* c) {
+    return c->unit_kind == QSTATE_UNIT_ROW ? static_cast<long long>(c->H) * c->dk : c->H;
+}
+long long groups_of(const qstate_cfg* c) {
+    return c->unit_kind == QSTATE_UNIT_ROW ? static_cast<long long>(c->H) * c->dk
+                                           : static_cast<long long>(c->H) * (c->dk / 32) * c->dv;
+}
+
+int validate(const qstate_cfg* c) {
+    if (!c) return fail(QSTATE_EINVAL, "cfg is NULL");
+    if (c->B < 1 || c->H < 1 || c->H > 1024) return fail(QSTATE_EINVAL, "need B >= 1 and 1 <= H <= 1024");
+    const bool shape_ok = (c->dk == 128 && c->dv == 128) || (c->dk == 128 && c->dv == 64) ||
+                          (c->dk == 64 && c->dv == 64);
+    if (!shape_ok) return fail(QSTATE_EINVAL, "unsupported (dk, dv) = (%d, %d)", c->dk, c->dv);
+    if (c->decay_kind != QSTATE_DECAY_ROW && c->decay_kind != QSTATE_DECAY_HEAD)
+        return fail(QSTATE_EINVAL, "bad decay_kind");
+    if (c->erase_kind != QSTATE_ERASE_DELTA && c->erase_kind != QSTATE_ERASE_NONE)
+        return fail(QSTATE_EINVAL, "bad erase_kind");
+    if (c->unit_kind != QSTATE_UNIT_ROW && c->unit_kind != QSTATE_UNIT_HEAD)
+        return fail(QSTATE_EINVAL, "bad unit_kind");
+    if (c->unit_kind == QSTATE_UNIT_HEAD && c->decay_kind != QSTATE_DECAY_HEAD)
+        return fail(QSTATE_EINVAL, "the head unit needs per-head decay");
+    if (c->unit_kind == QSTATE_UNIT_ROW && (c->group_heads < 1 || c->H % c->group_heads != 0))
+        return fail(QSTATE_EINVAL, "group_heads must divide H");
+    if (c->bbar_den < 1 || c->bbar_num < 0) return fail(QSTATE_EINVAL, "bad bbar fraction");
+    if (c->bmin < 0 || c->bmax > 16 || c->bmin > c->bmax) return fail(QSTATE_EINVAL, "need 0 <= bmin <= bmax <= 16");
+    const long long bits = static_cast<long long>(c->H) * c->dk * c->dv * c->bbar_num;
+    if (bits % (8LL * c->bbar_den) != 0) return fail(QSTATE_EINVAL, "budget is not a whole number of bytes");
+    const long long N = units_of(c);
+    if ((N * c->bbar_num) % c->bbar_den != 0) return fail(QSTATE_EINVAL, "units * bbar is not an integer");
+    const long long total = N * c->bbar_num / c->bbar_den;
+    if (N * c->bmin > total || N * c->bmax < total)
+        return fail(QSTATE_EBUDGET, "budget %lld bits per element sum outside [%lld, %lld]", total,
+                    N * c->bmin, N * c->bmax);
+    if (c->C < 1) return fail(QSTATE_EINVAL, "C must be >= 1");
+    if (c->fit_every < 1) return fail(QSTATE_EINVAL, "fit_every must be >= 1");
+    if (!(c->ema_span > 0.0f)) return fail(QSTATE_EINVAL, "ema_span must be > 0");
+    if (c->gate_bits < 0 || c->gate_bits > 8) return fail(QSTATE_EINVAL, "gate_bits must be in [0, 8]");
+    if (c->weight_kind != QSTATE_WEIGHT_OURS) return fail(QSTATE_EINVAL, "unsupported weight_kind");
+    return QSTATE_OK;
+}
+
+long long region_of(const qstate_cfg* c) {
+    return static_cast<long long>(c->H) * c->dk * c->dv * c->bbar_num / (8LL * c->bbar_den);
+}
+
+bool buf_ok(const qstate_buf* b) {
+    return b && b->payload && b->scales && b->widths && b->head_off && b->fidx;
+}
+
+cudaError_t launch_step_any(const qstate_cfg& c, int src_packed, int dst_packed, const StepParams& p,
+                            cudaStream_t st) {
+    if (c.dk == 128 && c.dv == 128) return launch_step_128x128(c, src_packed, dst_packed, p, st);
+    if (c.dk == 128 && c.dv == 64) return launch_step_128x64(c, src_packed, dst_packed, p, st);
+    return launch_step_64x64(c, src_packed, dst_packed, p, st);
+}
+
+StepParams base_params(const qstate_cfg* c, int* status) {
+    StepParams p;
+    std::memset(&p, 0, sizeof(p));
+    p.B = c->B;
+    p.H = c->H;
+    p.erase = c->erase_kind == QSTATE_ERASE_DELTA ? 1 : 0;
+    p.decay_row = c->decay_kind == QSTATE_DECAY_ROW ? 1 : 0;
+    p.fit_every = c->fit_every;
+    p.L = c->gate_bits > 0 ? (1 << c->gate_bits) : 0;
+    p.group_heads = c->group_heads;
+    p.region_bytes = region_of(c);
+    p.alpha = 2.0f / (c->ema_span + 1.0f);
+    p.status = status;
+    return p;
+}
+
+int check_inputs(const qstate_cfg* c, const qstate_inputs* x, int t_begin, int t_end, const float* o) {
+    if (!x || !x->q || !x->k || !x->v || !o) return fail(QSTATE_EINVAL, "null input or output pointer");
+    if (c->erase_kind == QSTATE_ERASE_DELTA && !x->beta) return fail(QSTATE_EINVAL, "beta is NULL");
+    if (x->s_code) {
+        if (c->gate_bits < 1 || !x->s_lut) return fail(QSTATE_EINVAL, "s_code needs gate_bits >= 1 and s_lut");
+    } else if (!x->s) {
+        return fail(QSTATE_EINVAL, "decay rates are NULL");
+    }
+    if (t_begin < 0 || t_end < t_begin || t_end > x->T) return fail(QSTATE_EINVAL, "bad token range");
+    return QSTATE_OK;
+}
+
+void set_inputs(StepParams& p, const qstate_inputs* x) {
+    p.T = x->T;
+    p.q = x->q;
+    p.k = x->k;
+    p.v = x->v;
+    p.s = x->s_code ? nullptr : x->s;
+    p.s_code = x->s_code;
+    p.s_lut = x->s_lut;
+    p.beta = x->beta;
+}
+
+int run_alloc(const qstate_cfg* c, const float* ms, const float* mr, const float* range, int uniform,
+              uint8_t* widths, uint32_t* head_off, int* status, cudaStream_t st) {
+    AllocParams a;
+    std::memset(&a, 0, sizeof(a));
+    a.B = c->B;
+    a.H = c->H;
+    a.dk = c->dk;
+    a.dv = c->dv;
+    a.units = static_cast<int>(units_of(c));
+    a.unit_row = c->unit_kind == QSTATE_UNIT_ROW ? 1 : 0;
+    a.group_heads = c->unit_kind == QSTATE_UNIT_ROW ? c->group_heads : 1;
+    a.bmin = c->bmin;
+    a.bmax = c->bmax;
+    a.total = units_of(c) * c->bbar_num / c->bbar_den;
+    a.uniform = uniform;
+    a.ema_s = ms;
+    a.ema_r = mr;
+    a.range = range;
+    a.widths = widths;
+    a.head_off = head_off;
+    a.status = status;
+    double fact = 1.0;
+    for (int k = 1; k <= 16; ++k) {
+        fact *= static_cast<double>(k);
+        a.e1[k] = static_cast<float>(1.0 / fact);
+    }
+    cudaError_t e = launch_alloc(a, st);
+    return e == cudaSuccess ? QSTATE_OK : cuda_fail(e, "allocation kernel");
+}
+
+}  // namespace
+
+extern "C" {
+
+int qstate_validate(const qstate_cfg* cfg) { return validate(cfg); }
+
+size_t qstate_region_bytes(const qstate_cfg* cfg) {
+    return validate(cfg) == QSTATE_OK ? static_cast<size_t>(region_of(cfg)) : 0;
+}
+
+size_t qstate_units(const qstate_cfg* cfg) {
+    return validate(cfg) == QSTATE_OK ? static_cast<size_t>(units_of(cfg)) : 0;
+}
+
+size_t qstate_scale_groups(const qstate_cfg* cfg) {
+    return validate(cfg) == QSTATE_OK ? static_cast<size_t>(groups_of(cfg)) : 0;
+}
+
+double qstate_bits_per_element(const qstate_cfg* cfg) {
+    if (validate(cfg) != QSTATE_OK) return 0.0;
+    const double bbar = static_cast<double>(cfg->bbar_num) / cfg->bbar_den;
+    int wbits = 0;
+    while ((1 << wbits) < cfg->bmax - cfg->bmin + 1) ++wbits;
+    if (cfg->unit_kind == QSTATE_UNIT_ROW) return bbar + (16.0 + wbits) / cfg->dv;
+    return bbar + 0.5 + static_cast<double>(wbits) / (static_cast<double>(cfg->dk) * cfg->dv);
+}
+
+int qstate_init(const qstate_cfg* cfg, qstate_buf* a, qstate_buf* b, void* stream) {
+    int rc = validate(cfg);
+    if (rc) return rc;
+    if (!buf_ok(a) || !buf_ok(b)) return fail(QSTATE_EINVAL, "null buffer pointer");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaError_t e;
+    int* status = status_word(&e);
+    if (!status) return cuda_fail(e, "status word");
+    rc = run_alloc(cfg, nullptr, nullptr, nullptr, 1, a->widths, a->head_off, status, st);
+    if (rc) return rc;
+    const size_t nw = static_cast<size_t>(cfg->B) * units_of(cfg);
+    e = cudaMemcpyAsync(b->widths, a->widths, nw, cudaMemcpyDeviceToDevice, st);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(b->head_off, a->head_off, sizeof(uint32_t) * cfg->B * cfg->H,
+                            cudaMemcpyDeviceToDevice, st);
+    if (e != cudaSuccess) return cuda_fail(e, "copy of initial widths");
+    StepParams p = base_params(cfg, status);
+    p.fit_every = 1;
+    p.out_payload = a->payload;
+    p.out_scales = a->scales;
+    p.out_widths = a->widths;
+    p.out_head_off = a->head_off;
+    p.out_fidx = a->fidx;
+    e = launch_step_any(*cfg, 0, 1, p, st);   // dense zero state -> packed
+    return e == cudaSuccess ? QSTATE_OK : cuda_fail(e, "pack kernel");
+}
+
+int qstate_alloc_bits(const qstate_cfg* cfg, const qstate_stats* stats, uint8_t* widths_out,
+                      uint32_t* head_off_out, void* stream) {
+    int rc = validate(cfg);
+    if (rc) return rc;
+    if (!stats || !stats->ema_s || !stats->ema_r || !widths_out || !head_off_out ||
+        (cfg->unit_kind == QSTATE_UNIT_ROW && !stats->range))
+        return fail(QSTATE_EINVAL, "null pointer");
+    cudaError_t e;
+    int* status = status_word(&e);
+    if (!status) return cuda_fail(e, "status word");
+    return run_alloc(cfg, stats->ema_s, stats->ema_r, stats->range, 0, widths_out, head_off_out,
+                     status, static_cast<cudaStream_t>(stream));
+}
+
+int qstate_pack(const qstate_cfg* cfg, const float* S, qstate_buf* out, float* range_out, void* stream) {
+    int rc = validate(cfg);
+    if (rc) return rc;
+    if (!S || !buf_ok(out)) return fail(QSTATE_EINVAL, "null pointer");
+    cudaError_t e;
+    int* status = status_word(&e);
+    if (!status) return cuda_fail(e, "status word");
+    StepParams p = base_params(cfg, status);
+    p.fit_every = 1;
+    p.dense_in = S;
+    p.out_payload = out->payload;
+    p.out_scales = out->scales;
+    p.out_widths = out->widths;
+    p.out_head_off = out->head_off;
+    p.out_fidx = out->fidx;
+    p.range = range_out;
+    e = launch_step_any(*cfg, 0, 1, p, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? QSTATE_OK : cuda_fail(e, "pack kernel");
+}
+
+int qstate_unpack(const qstate_cfg* cfg, const qstate_buf* in, float* S_out, void* stream) {
+    int rc = validate(cfg);
+    if (rc) return rc;
+    if (!S_out || !buf_ok(in)) return fail(QSTATE_EINVAL, "null pointer");
+    cudaError_t e;
+    int* status = status_word(&e);
+    if (!status) return cuda_fail(e, "status word");
+    StepParams p = base_params(cfg, status);
+    p.in_payload = in->payload;
+    p.in_scales = in->scales;
+    p.in_widths = in->widths;
+    p.in_head_off = in->head_off;
+    p.in_fidx = in->fidx;
+    p.dense_out = S_out;
+    e = launch_step_any(*cfg, 1, 0, p, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? QSTATE_OK : cuda_fail(e, "unpack kernel");
+}
+
+int qstate_quant_decay(const qstate_cfg* cfg, const float* s, int32_t T, uint8_t* code_out,
+                       float* lut_out, float* thr_out, void* stream) {
+    int rc = validate(cfg);
+    if (rc) return rc;
+    if (cfg->gate_bits < 1) return fail(QSTATE_EINVAL, "gate_bits must be >= 1");
+    if (!s || !code_out || !lut_out || !thr_out || T < 1) return fail(QSTATE_EINVAL, "null pointer or T < 1");
+    cudaError_t e;
+    int* status = status_word(&e);
+    if (!status) return cuda_fail(e, "status word");
+    const int nchan = cfg->decay_kind == QSTATE_DECAY_ROW ? cfg->H * cfg->dk : cfg->H;
+    const long long count = static_cast<long long>(cfg->B) * T;
+    e = launch_quant_decay(s, count, nchan, cfg->gate_bits, code_out, lut_out, thr_out, status,
+                           static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? QSTATE_OK : cuda_fail(e, "decay quantiser");
+}
+
+int qstate_step(const qstate_cfg* cfg, qstate_buf* in, qstate_buf* out, const qstate_inputs* x,
+                int32_t t_begin, int32_t t_end, int32_t w_index, float* o, qstate_stats* stats,
+                void* stream) {
+    int rc = validate(cfg);
+    if (rc) return rc;
+    if (!buf_ok(in) || !buf_ok(out)) return fail(QSTATE_EINVAL, "null buffer pointer");
+    if (!stats || !stats->ema_s || !stats->ema_r || (cfg->unit_kind == QSTATE_UNIT_ROW && !stats->range))
+        return fail(QSTATE_EINVAL, "null statistics pointer");
+    if ((rc = check_inputs(cfg, x, t_begin, t_end, o))) return rc;
+    if (t_end - t_begin > cfg->C || t_end == t_begin)
+        return fail(QSTATE_EINVAL, "a write-back interval holds 1..C tokens");
+    if (x->s_code && cfg->gate_bits < 1) return fail(QSTATE_EINVAL, "s_code needs gate_bits");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaError_t e;
+    int* status = status_word(&e);
+    if (!status) return cuda_fail(e, "status word");
+    StepParams p = base_params(cfg, status);
+    set_inputs(p, x);
+    p.t_begin = t_begin;
+    p.t_end = t_end;
+    p.w_index = w_index;
+    p.in_payload = in->payload;
+    p.in_scales = in->scales;
+    p.in_widths = in->widths;
+    p.in_head_off = in->head_off;
+    p.in_fidx = in->fidx;
+    p.out_payload = out->payload;
+    p.out_scales = out->scales;
+    p.out_widths = out->widths;
+    p.out_head_off = out->head_off;
+    p.out_fidx = out->fidx;
+    p.o = o;
+    p.ema_s = stats->ema_s;
+    p.ema_r = stats->ema_r;
+    p.range = stats->range;
+    e = launch_step_any(*cfg, 1, 1, p, st);
+    if (e != cudaSuccess) return cuda_fail(e, "write-back kernel");
+    return run_alloc(cfg, stats->ema_s, stats->ema_r, stats->range, 0, in->widths, in->head_off,
+                     status, st);
+}
+
+int qstate_scan(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong, const qstate_inputs* x,
+                int32_t t_begin, int32_t t_end, int32_t w_index0, float* o, qstate_stats* stats,
+                int32_t* final_in_pong, void* stream) {
+    int rc = validate(cfg);
+    if (rc) return rc;
+    if ((rc = check_inputs(cfg, x, t_begin, t_end, o))) return rc;
+    qstate_buf* src = ping;
+    qstate_buf* dst = pong;
+    int in_pong = 0;
+    int w = w_index0;
+    for (int t0 = t_begin; t0 < t_end; t0 += cfg->C) {
+        const int t1 = t0 + cfg->C < t_end ? t0 + cfg->C : t_end;
+        rc = qstate_step(cfg, src, dst, x, t0, t1, w++, o, stats, stream);
+        if (rc) return rc;
+        qstate_buf* tmp = src;
+        src = dst;
+        dst = tmp;
+        in_pong ^= 1;
+    }
+    if (final_in_pong) *final_in_pong = in_pong;
+    return QSTATE_OK;
+}
+
+int qstate_scan_fp32(const qstate_cfg* cfg, float* S, const qstate_inputs* x, int32_t t_begin,
+                     int32_t t_end, float* o, void* stream) {
+    int rc = validate(cfg);
+    if (rc) return rc;
+    if (!S) return fail(QSTATE_EINVAL, "S is NULL");
+    if ((rc = check_inputs(cfg, x, t_begin, t_end, o))) return rc;
+    cudaError_t e;
+    int* status = status_word(&e);
+    if (!status) return cuda_fail(e, "status word");
+    StepParams p = base_params(cfg, status);
+    set_inputs(p, x);
+    p.dense_in = S;
+    p.dense_out = S;
+    p.o = o;
+    for (int t0 = t_begin; t0 < t_end; t0 += cfg->C) {
+        p.t_begin = t0;
+        p.t_end = t0 + cfg->C < t_end ? t0 + cfg->C : t_end;
+        e = launch_step_any(*cfg, 0, 0, p, static_cast<cudaStream_t>(stream));
+        if (e != cudaSuccess) return cuda_fail(e, "fp32 write-back kernel");
+    }
+    return QSTATE_OK;
+}
+
+int qstate_check(void* stream) {
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+    int* status = status_word(&e);
+    if (!status) return cuda_fail(e, "status word");
+    int v = 0;
+    e = cudaMemcpy(&v, status, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "status read");
+    if (v != 0) {
+        const int zero = 0;
+        e = cudaMemcpy(status, &zero, sizeof(int), cudaMemcpyHostToDevice);
+        if (e != cudaSuccess) return cuda_fail(e, "status clear");
+        return fail(QSTATE_EDEVICE, "device status 0x%x:%s%s", v,
+                    (v & QS_DEV_LAYOUT) ? " inconsistent widths/offsets" : "",
+                    (v & QS_DEV_RATE) ? " decay rate not positive/finite" : "");
+    }
+    return QSTATE_OK;
+}
+
+const char* qstate_last_error(void) { return g_err; }
+
+}  // extern "C"

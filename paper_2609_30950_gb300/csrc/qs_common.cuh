@@ -1,0 +1,135 @@
+// qs_common.cuh -- device helpers shared by the libqstate kernels (sm_103a).
+//
+// Floating-point operations that decide an integer (a code, a fitted factor, a width) are
+// written with explicit IEEE intrinsics (__fmul_rn, __fadd_rn, __frcp_rn, ...) so that the
+// compiler cannot contract them into FMAs: the stored format is then reproducible.
+#pragma once
+
+#include <cuda_fp16.h>
+#include <stdint.h>
+
+#include "qs_internal.h"
+
+namespace qs {
+
+constexpr unsigned kFull = 0xffffffffu;
+// 1.5 * 2^23: y + kMagic rounds y to an integer (round-half-even) for |y| < 2^22, and the
+// result's low mantissa bits hold that integer offset by 2^22.
+constexpr float kMagic = 12582912.0f;
+constexpr uint32_t kMagicBits = 0x4B400000u;
+// 2^23: the float with bits 0x4B000000 | u equals 2^23 + u for u < 2^23.
+constexpr uint32_t kTwo23Bits = 0x4B000000u;
+
+// Record a QS_DEV_* condition in the status word (one per device, see qs_api.cu).
+__device__ __forceinline__ void raise_status(int* status, int bits) {
+    if (status) atomicOr(status, bits);
+}
+
+// ---- FP16 scale (Sec. 3, "Levels and storage") -------------------------------------------
+// Round to binary16 (nearest even), magnitudes saturated at 65504, returned as float.
+__device__ __forceinline__ float f16_round(float x) {
+    x = fminf(fmaxf(x, -65504.0f), 65504.0f);
+    return __half2float(__float2half_rn(x));
+}
+__device__ __forceinline__ uint16_t f16_bits(float x) {
+    x = fminf(fmaxf(x, -65504.0f), 65504.0f);
+    return __half_as_ushort(__float2half_rn(x));
+}
+__device__ __forceinline__ float f16_value(uint16_t u) { return __half2float(__ushort_as_half(u)); }
+
+// The 16 candidate range factors f_k = (5 + k) / 20 on [1/4, 1] (Sec. 3), correctly rounded.
+__device__ __forceinline__ float fit_factor(int k) {
+    return __fdiv_rn(static_cast<float>(5 + k), 20.0f);
+}
+
+// Candidate step for factor f: Delta = FP16(fl(fl(f R) * fl(1/n))).
+__device__ __forceinline__ float cand_step(float f, float R, float inv_n) {
+    return f16_round(__fmul_rn(__fmul_rn(f, R), inv_n));
+}
+__device__ __forceinline__ float step_rcp(float D) { return D == 0.0f ? 0.0f : __frcp_rn(D); }
+
+// clamp(rint(x * inv), -n, n) in the magic domain: returns kMagic + q (exact integer float).
+__device__ __forceinline__ float code_magic(float x, float inv, float lo, float hi) {
+    float t = __fadd_rn(__fmul_rn(x, inv), kMagic);
+    return fminf(fmaxf(t, lo), hi);
+}
+
+// ---- warp reductions ----------------------------------------------------------------------
+__device__ __forceinline__ float warp_absmax(float v) {
+    unsigned m = __reduce_max_sync(kFull, __float_as_uint(fabsf(v)));
+    return __uint_as_float(m);
+}
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+    return v;
+}
+
+// ---- row bitstream (Sec. 3 storage; this library's bit order) ------------------------------
+// A lane owning CPL consecutive elements of a row reads its CPL*w bits starting at row bit
+// lane*CPL*w.  `row` is 8-byte aligned shared memory followed by >= 12 readable bytes.
+template <int CPL>
+__device__ __forceinline__ void extract_codes(const uint8_t* row, int lane, int w,
+                                              uint32_t (&u)[CPL]) {
+    const uint32_t* words = reinterpret_cast<const uint32_t*>(row);
+    const int P = lane * CPL * w;
+    const int idx = P >> 5, sh = P & 31;
+    const uint32_t mask = (w >= 32) ? 0xffffffffu : ((1u << w) - 1u);
+    if (CPL * w <= 32) {
+        uint32_t chunk = __funnelshift_r(words[idx], words[idx + 1], sh);
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) u[c] = (chunk >> (c * w)) & mask;
+    } else {
+        uint32_t lo = __funnelshift_r(words[idx], words[idx + 1], sh);
+        uint32_t hi = __funnelshift_r(words[idx + 1], words[idx + 2], sh);
+        uint64_t chunk = (static_cast<uint64_t>(hi) << 32) | lo;
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) u[c] = static_cast<uint32_t>(chunk >> (c * w)) & mask;
+    }
+}
+
+// Write the row's codes.  Lanes form groups of G = CPL-lane chunks whose combined width is a
+// whole number of bytes; the group's first lane writes them.  Every byte of the row is
+// written exactly once (no zero fill needed).  All 32 lanes must call this.
+template <int CPL>
+__device__ __forceinline__ void store_codes(uint8_t* row, int lane, int w, const uint32_t (&u)[CPL]) {
+    uint64_t chunk = 0;
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) chunk |= static_cast<uint64_t>(u[c]) << (c * w);
+    const int cb = CPL * w;                     // bits per lane
+    // smallest G (1, 2 or 4) with G * cb a multiple of 8
+    const int G = (cb % 8 == 0) ? 1 : ((2 * cb) % 8 == 0 ? 2 : 4);
+    // gather the group's chunks into a 128-bit value (lo, hi)
+    uint64_t lo = chunk, hi = 0;
+#pragma unroll
+    for (int g = 1; g < 4; ++g) {
+        uint64_t other = __shfl_down_sync(kFull, chunk, g);
+        if (g < G) {
+            const int s = g * cb;               // 1 <= s < 128
+            if (s < 64) {
+                lo |= other << s;
+                hi |= other >> (64 - s);
+            } else {
+                hi |= other << (s - 64);
+            }
+        }
+    }
+    if ((lane % G) == 0) {
+        const int nbytes = (G * cb) >> 3;
+        uint8_t* dst = row + (lane / G) * nbytes;
+        for (int k = 0; k < nbytes; ++k) {
+            uint64_t src = (k < 8) ? lo : hi;
+            dst[k] = static_cast<uint8_t>(src >> ((k & 7) * 8));
+        }
+    }
+}
+
+// Dequantised value of code u at width w (Sec. 3 levels): w >= 2 -> (u - n) Delta,
+// w = 1 -> +-m, w = 0 -> 0.  nf2 = 2^23 + n (exact).
+__device__ __forceinline__ float dequant(uint32_t u, int w, float D, float nf2) {
+    if (w >= 2) return __fmul_rn(__fsub_rn(__uint_as_float(kTwo23Bits | u), nf2), D);
+    if (w == 1) return u ? -D : D;
+    return 0.0f;
+}
+
+}  // namespace qs

@@ -1,0 +1,83 @@
+// qs_internal.h -- kernel parameter blocks and launch entry points inside libqstate.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/qstate.h"
+
+namespace qs {
+
+// device status bits
+enum : int {
+    QS_DEV_LAYOUT = 1,  // widths/offsets inconsistent with the region
+    QS_DEV_RATE = 2,    // a decay rate is not a positive finite number
+};
+
+constexpr int kNFit = 16;
+
+// Parameters of the fused write-back kernel.  src/dst are packed or dense depending on the
+// kernel instantiation.
+struct StepParams {
+    int B, H, T;
+    int t_begin, t_end, w_index;
+    int erase;        // 1: delta rule (a = beta k, w = beta 1); 0: a = 0, w = 1
+    int decay_row;    // 1: per-row rates; 0: per-head rates
+    int fit_every;
+    int L;            // 2^gate_bits (0 when rates are FP32)
+    int group_heads;
+    long long region_bytes;
+    int stage_bytes;  // shared-memory staging capacity for one head's rows (dk dv bmax / 8)
+    float alpha;      // EMA weight 2 / (span + 1)
+    // packed source / destination
+    const uint8_t* in_payload;
+    const uint16_t* in_scales;
+    const uint8_t* in_widths;
+    const uint32_t* in_head_off;
+    const uint8_t* in_fidx;
+    uint8_t* out_payload;
+    uint16_t* out_scales;
+    const uint8_t* out_widths;
+    const uint32_t* out_head_off;
+    uint8_t* out_fidx;
+    // dense source / destination (B, H, dk, dv); src may be null (= zero state)
+    const float* dense_in;
+    float* dense_out;
+    // token inputs
+    const float* q;
+    const float* k;
+    const float* v;
+    const float* s;
+    const uint8_t* s_code;
+    const float* s_lut;
+    const float* beta;
+    float* o;
+    // statistics (may be null when there are no tokens)
+    float* ema_s;
+    float* ema_r;
+    float* range;
+    int* status;
+};
+
+struct AllocParams {
+    int B, H, dk, dv, units, unit_row, group_heads, bmin, bmax;
+    long long total;   // sum of widths per batch element
+    int uniform;       // 1: ignore statistics, equal weights (initial widths)
+    const float* ema_s;
+    const float* ema_r;
+    const float* range;
+    uint8_t* widths;
+    uint32_t* head_off;
+    int* status;
+    float e1[17];      // 1/k! (FP64 -> FP32) for the expm1 series, k = 1..16
+};
+
+// launchers (return cudaError_t of the launch)
+cudaError_t launch_step(const qstate_cfg& cfg, int src_packed, int dst_packed,
+                        const StepParams& p, cudaStream_t stream);
+cudaError_t launch_alloc(const AllocParams& p, cudaStream_t stream);
+cudaError_t launch_quant_decay(const float* s, long long count, int nchan, int g,
+                               uint8_t* codes, float* lut, float* thr, int* status,
+                               cudaStream_t stream);
+
+}  // namespace qs

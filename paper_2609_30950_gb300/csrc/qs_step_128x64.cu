@@ -1,0 +1,9 @@
+// qs_step_128x64.cu -- write-back kernel instantiations for dk = 128, dv = 64.
+#include "qs_step_impl.cuh"
+
+namespace qs {
+cudaError_t launch_step_128x64(const qstate_cfg& cfg, int src_packed, int dst_packed,
+                            const StepParams& p, cudaStream_t stream) {
+    return launch_step_shape<128, 64>(cfg, src_packed, dst_packed, p, stream);
+}
+}  // namespace qs

@@ -1,0 +1,571 @@
+// qs_step_impl.cuh -- the fused write-back kernel of libqstate (sm_103a).
+//
+// One CTA per (batch element, head), 8 warps.  Warp w owns key rows [w*RPW, (w+1)*RPW); lane
+// l owns value columns [l*CPL, (l+1)*CPL) of each of them, so one row is handled by one warp
+// and its bit width is warp-uniform.  The head's FP32 state lives in registers for the whole
+// write-back interval:
+//   1. metadata (widths -> row offsets by prefix sums, Sec. 3 "Prefix sums of widths give row
+//      offsets"), layout check;
+//   2. the head's packed rows are staged in shared memory with 16-byte (dv = 128) or 8-byte
+//      (dv = 64) vector loads;
+//   3. unpack + dequantise (Sec. 3 levels);
+//   4. per token (Eq. 1): decay, fused reductions p = (beta k)^T S', r = q^T S' (per-lane
+//      partials over the warp's rows, then across warps in shared memory), delta update,
+//      readout o = S^T q = r + u (k . q) before quantisation (Sec. 2), EMA statistics (Sec. 3);
+//   5. range, fitted FP16 scale (16 candidates, Sec. 3), codes, repack to shared memory and a
+//      vector store of the head's new region.
+// The same template serves pack (dense -> packed, no tokens), unpack (packed -> dense) and the
+// unquantised reference path (dense -> dense).
+#pragma once
+
+#include <type_traits>
+
+#include "qs_common.cuh"
+
+namespace qs {
+
+template <int DK, int DV, bool HEAD>
+struct alignas(16) StepSmem {
+    static constexpr int NW = 8;
+    static constexpr int NSG = HEAD ? (DK / 32) * DV : DK;
+    float k[DK], q[DK], d[DK];
+    float v[DV], u[DV];
+    float red[2][NW][DV];                 // p and r partials per warp
+    float scale_in[NSG];                  // source steps / means (float)
+    float ms[DK], mr[DK];                 // EMA statistics (head unit uses [0])
+    float fit_red[HEAD ? NW * 4 * DV : 1];// head unit: partial SSEs, 4 candidates per round
+    float colmax[HEAD ? NW * DV : 1];     // head unit: per-warp column maxima / sums
+    float wsum[2][NW];                    // per-warp partial k.q and |k|^2
+    int off_in[DK + 1], off_out[DK + 1];  // row byte offsets inside the head (+ total)
+    uint8_t w_in[DK], w_out[DK];
+    uint8_t fidx_in[NSG];
+    int flag;
+};
+
+// Sum 16 per-lane values over the warp by recursive halving; lane l ends with the total of
+// value index (l >> 1) & 15.
+__device__ __forceinline__ float reduce16(float (&v)[16], int lane) {
+#pragma unroll
+    for (int st = 0; st < 4; ++st) {
+        const int half = 8 >> st;
+        const int off = 16 >> st;
+        const bool upper = (lane & off) != 0;
+#pragma unroll
+        for (int i = 0; i < half; ++i) {
+            float send = upper ? v[i] : v[i + half];
+            float keep = upper ? v[i + half] : v[i];
+            v[i] = keep + __shfl_xor_sync(kFull, send, off);
+        }
+    }
+    return v[0] + __shfl_xor_sync(kFull, v[0], 1);
+}
+
+template <int CPL>
+struct RowVals {
+    float v[CPL];
+};
+struct RowOut {
+    float R;
+    unsigned scale;
+    int fidx;
+};
+
+// Row unit write-back of one row (Sec. 3, "Levels and storage"): range R = max |x|, fitted
+// FP16 step (16 candidates, smallest squared error, ties to the larger factor) or 1-bit mean,
+// codes, and the row's bytes written to `row` (shared memory).  Called by all 32 lanes.
+template <int CPL, int DV>
+__device__ __noinline__ RowOut quantise_row(RowVals<CPL> xv, int w, int lane, bool refit,
+                                            int fidx_in, uint8_t* row) {
+    float amax = 0.0f;
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) amax = fmaxf(amax, fabsf(xv.v[c]));
+    RowOut out;
+    out.R = warp_absmax(amax);
+    out.scale = 0;
+    out.fidx = fidx_in;
+    uint32_t u[CPL];
+    if (w == 1) {
+        float sa = 0.0f;
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) sa += fabsf(xv.v[c]);
+        sa = warp_sum(sa);
+        out.scale = f16_bits(__fdiv_rn(sa, static_cast<float>(DV)));
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) u[c] = xv.v[c] < 0.0f ? 1u : 0u;
+    } else if (w >= 2) {
+        const int n = (1 << (w - 1)) - 1;
+        const float nf = static_cast<float>(n);
+        const float inv_n = __frcp_rn(nf);
+        const float R = out.R;
+        if (R == 0.0f) {
+            if (refit) out.fidx = kNFit - 1;
+#pragma unroll
+            for (int c = 0; c < CPL; ++c) u[c] = static_cast<uint32_t>(n);
+        } else {
+            if (refit) {
+                // lane l prepares candidate l & 15; every lane scores all 16 on its elements
+                const float Dl = cand_step(fit_factor(lane & 15), R, inv_n);
+                const float il = step_rcp(Dl);
+                float sse[16];
+#pragma unroll
+                for (int k = 0; k < 16; ++k) {
+                    const float D = __shfl_sync(kFull, Dl, k);
+                    const float inv = __shfl_sync(kFull, il, k);
+                    float acc = 0.0f;
+#pragma unroll
+                    for (int c = 0; c < CPL; ++c) {
+                        const float a = fabsf(xv.v[c]);
+                        const float tq = fminf(__fadd_rn(__fmul_rn(a, inv), kMagic), kMagic + nf);
+                        const float e = fmaf(-__fsub_rn(tq, kMagic), D, a);
+                        acc = fmaf(e, e, acc);
+                    }
+                    sse[k] = acc;
+                }
+                const float tot = reduce16(sse, lane);
+                const unsigned sb = __float_as_uint(tot);
+                const unsigned mn = __reduce_min_sync(kFull, sb);
+                const unsigned best = __reduce_max_sync(kFull, sb == mn ? ((lane >> 1) & 15) + 1 : 0u);
+                out.fidx = static_cast<int>(best) - 1;
+            }
+            const float D = cand_step(fit_factor(out.fidx), R, inv_n);
+            const float inv = step_rcp(D);
+            out.scale = f16_bits(D);
+#pragma unroll
+            for (int c = 0; c < CPL; ++c) {
+                const float tq = code_magic(xv.v[c], inv, kMagic - nf, kMagic + nf);
+                u[c] = __float_as_uint(tq) - (kMagicBits - static_cast<uint32_t>(n));
+            }
+        }
+    } else {
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) u[c] = 0u;
+    }
+    store_codes<CPL>(row, lane, w, u);
+    return out;
+}
+
+template <int DK, int DV, bool HEAD, bool SRC_PACKED, bool DST_PACKED>
+__global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
+    constexpr int NW = 8, RPW = DK / NW, CPL = DV / 32;
+    using Sm = StepSmem<DK, DV, HEAD>;
+    constexpr int NSG = Sm::NSG;
+    extern __shared__ __align__(16) uint8_t smem_raw[];
+    Sm& sm = *reinterpret_cast<Sm*>(smem_raw);
+    uint8_t* pay = smem_raw + sizeof(Sm);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int bh = blockIdx.x, b = bh / p.H, h = bh - b * p.H;
+    const size_t ubase = HEAD ? static_cast<size_t>(bh) : static_cast<size_t>(bh) * DK;
+    const size_t gbase = static_cast<size_t>(bh) * NSG;
+    const bool has_tokens = p.t_end > p.t_begin;
+    const bool stats = has_tokens && p.ema_s != nullptr;
+
+    // ---- 1. metadata ---------------------------------------------------------------------
+    if (tid == 0) sm.flag = 0;
+    if (SRC_PACKED) {
+        for (int i = tid; i < DK; i += 256) sm.w_in[i] = HEAD ? p.in_widths[bh] : p.in_widths[ubase + i];
+        for (int g = tid; g < NSG; g += 256) sm.scale_in[g] = f16_value(p.in_scales[gbase + g]);
+    }
+    if (DST_PACKED) {
+        for (int i = tid; i < DK; i += 256) sm.w_out[i] = HEAD ? p.out_widths[bh] : p.out_widths[ubase + i];
+        for (int g = tid; g < NSG; g += 256) sm.fidx_in[g] = p.in_fidx ? p.in_fidx[gbase + g] : 15;
+    }
+    if (stats) {
+        if (!HEAD) {
+            for (int i = tid; i < DK; i += 256) {
+                sm.ms[i] = p.ema_s[ubase + i];
+                sm.mr[i] = p.ema_r[ubase + i];
+            }
+        } else if (tid == 0) {
+            sm.ms[0] = p.ema_s[ubase];
+            sm.mr[0] = p.ema_r[ubase];
+        }
+    }
+    __syncthreads();
+    if ((warp == 0 && SRC_PACKED) || (warp == 1 && DST_PACKED)) {
+        const uint8_t* wa = warp == 0 ? sm.w_in : sm.w_out;
+        int* off = warp == 0 ? sm.off_in : sm.off_out;
+        constexpr int PER = DK / 32;
+        int loc[PER];
+        int sum = 0;
+        bool bad = false;
+#pragma unroll
+        for (int j = 0; j < PER; ++j) {
+            const int w = wa[lane * PER + j];
+            bad |= (w > 16);
+            loc[j] = sum;
+            sum += w * (DV / 8);
+        }
+        int incl = sum;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int n = __shfl_up_sync(kFull, incl, o);
+            if (lane >= o) incl += n;
+        }
+        const int excl = incl - sum;
+#pragma unroll
+        for (int j = 0; j < PER; ++j) off[lane * PER + j] = excl + loc[j];
+        const int total = __shfl_sync(kFull, incl, 31);
+        bad = __any_sync(kFull, bad);
+        const long long hoff = warp == 0 ? p.in_head_off[bh] : p.out_head_off[bh];
+        const int align = (DV == 128) ? 16 : 8;
+        if (lane == 0) {
+            off[DK] = total;
+            if (bad || hoff + total > p.region_bytes || (hoff % align) != 0 || total > p.stage_bytes)
+                atomicExch(&sm.flag, 1);
+        }
+    }
+    __syncthreads();
+    if (sm.flag) {
+        if (tid == 0) raise_status(p.status, QS_DEV_LAYOUT);
+        return;
+    }
+
+    // ---- 2. stage the source rows in shared memory ----------------------------------------
+    using Vec = typename std::conditional<DV == 128, uint4, uint2>::type;
+    if (SRC_PACKED) {
+        const int nbytes = sm.off_in[DK];
+        const Vec* src = reinterpret_cast<const Vec*>(
+            p.in_payload + static_cast<size_t>(b) * p.region_bytes + p.in_head_off[bh]);
+        Vec* dst = reinterpret_cast<Vec*>(pay);
+        const int nv = nbytes / static_cast<int>(sizeof(Vec));
+        for (int i = tid; i < nv; i += 256) dst[i] = __ldg(src + i);
+        if (tid < 4) reinterpret_cast<uint32_t*>(pay + nbytes)[tid] = 0u;
+        __syncthreads();
+    }
+
+    // ---- 3. unpack + dequantise into registers ---------------------------------------------
+    float x[RPW][CPL];
+#pragma unroll
+    for (int r = 0; r < RPW; ++r) {
+        const int i = warp * RPW + r;
+        if (SRC_PACKED) {
+            const int w = sm.w_in[i];
+            uint32_t u[CPL];
+            extract_codes<CPL>(pay + sm.off_in[i], lane, w, u);
+            const float nf2 = 8388608.0f + static_cast<float>(w >= 2 ? (1 << (w - 1)) - 1 : 0);
+#pragma unroll
+            for (int c = 0; c < CPL; ++c) {
+                const float D = HEAD ? sm.scale_in[(i >> 5) * DV + lane * CPL + c] : sm.scale_in[i];
+                x[r][c] = dequant(u[c], w, D, nf2);
+            }
+        } else if (p.dense_in != nullptr) {
+            const float* src = p.dense_in + (static_cast<size_t>(bh) * DK + i) * DV + lane * CPL;
+            if (CPL == 4) {
+                const float4 t = *reinterpret_cast<const float4*>(src);
+                x[r][0] = t.x; x[r][1] = t.y; x[r][CPL > 2 ? 2 : 0] = t.z; x[r][CPL > 3 ? 3 : 0] = t.w;
+            } else {
+                const float2 t = *reinterpret_cast<const float2*>(src);
+                x[r][0] = t.x; x[r][1] = t.y;
+            }
+        } else {
+#pragma unroll
+            for (int c = 0; c < CPL; ++c) x[r][c] = 0.0f;
+        }
+    }
+    if (SRC_PACKED) __syncthreads();   // the staging buffer is reused for the output rows
+
+    // ---- 4. tokens of this write-back interval (Eq. 1) --------------------------------------
+    for (int t = p.t_begin; t < p.t_end; ++t) {
+        const size_t tok = (static_cast<size_t>(b) * p.T + t) * p.H + h;
+        const float beta = p.erase ? __ldg(p.beta + tok) : 1.0f;
+        float rate_h = 0.0f;
+        if (!p.decay_row)
+            rate_h = p.s_code ? __ldg(p.s_lut + static_cast<size_t>(h) * p.L +
+                                      min(static_cast<int>(p.s_code[tok]), p.L - 1))
+                              : __ldg(p.s + tok);
+        if (tid < DK) {
+            const int i = tid;
+            const float kk = __ldg(p.k + tok * DK + i), qq = __ldg(p.q + tok * DK + i);
+            sm.k[i] = kk;
+            sm.q[i] = qq;
+            float rate = rate_h;
+            if (p.decay_row)
+                rate = p.s_code ? __ldg(p.s_lut + (static_cast<size_t>(h) * DK + i) * p.L +
+                                        min(static_cast<int>(p.s_code[tok * DK + i]), p.L - 1))
+                                : __ldg(p.s + tok * DK + i);
+            if (!(rate > 0.0f) || !(rate < INFINITY)) raise_status(p.status, QS_DEV_RATE);
+            sm.d[i] = expf(-rate);
+            if (stats && !HEAD) {   // Sec. 3 statistics per row
+                const float xs = -expm1f(-2.0f * rate);
+                const float xr = p.erase ? __fmul_rn(__fmul_rn(beta, __fsub_rn(2.0f, beta)), __fmul_rn(kk, kk)) : 0.0f;
+                if (t == 0) {
+                    sm.ms[i] = xs;
+                    sm.mr[i] = xr;
+                } else {
+                    sm.ms[i] = __fadd_rn(sm.ms[i], __fmul_rn(p.alpha, __fsub_rn(xs, sm.ms[i])));
+                    sm.mr[i] = __fadd_rn(sm.mr[i], __fmul_rn(p.alpha, __fsub_rn(xr, sm.mr[i])));
+                }
+            }
+            const float kq = warp_sum(kk * qq);
+            const float k2 = warp_sum(kk * kk);
+            if (lane == 0) {
+                sm.wsum[0][warp] = kq;
+                sm.wsum[1][warp] = k2;
+            }
+        }
+        if (tid < DV) sm.v[tid] = __ldg(p.v + tok * DV + tid);
+        __syncthreads();
+
+        // decay and per-lane partial reductions over the warp's rows
+        float pp[CPL], rr[CPL];
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) pp[c] = rr[c] = 0.0f;
+#pragma unroll
+        for (int r = 0; r < RPW; ++r) {
+            const int i = warp * RPW + r;
+            const float d = sm.d[i];
+            const float a = __fmul_rn(beta, sm.k[i]);   // erase vector a = beta k
+            const float qi = sm.q[i];
+#pragma unroll
+            for (int c = 0; c < CPL; ++c) {
+                x[r][c] = __fmul_rn(x[r][c], d);
+                pp[c] = fmaf(x[r][c], a, pp[c]);
+                rr[c] = fmaf(x[r][c], qi, rr[c]);
+            }
+        }
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) {
+            sm.red[0][warp][lane * CPL + c] = pp[c];
+            sm.red[1][warp][lane * CPL + c] = rr[c];
+        }
+        __syncthreads();
+        if (tid < DV) {
+            const int j = tid;
+            float P = 0.0f, Rr = 0.0f, kq = 0.0f;
+#pragma unroll
+            for (int w = 0; w < NW; ++w) {
+                P += sm.red[0][w][j];
+                Rr += sm.red[1][w][j];
+            }
+#pragma unroll
+            for (int w = 0; w < DK / 32; ++w) kq += sm.wsum[0][w];
+            const float vj = sm.v[j];
+            // S = S' - k (a^T S') + k (w o v)^T:  u = beta v - p (delta rule), u = v (no erase)
+            const float u = p.erase ? __fsub_rn(__fmul_rn(beta, vj), P) : vj;
+            sm.u[j] = u;
+            p.o[tok * DV + j] = fmaf(u, kq, Rr);   // o = S^T q = S'^T q + u (k . q)
+        }
+        if (stats && HEAD && tid == 0) {   // Sec. 3 statistics per head
+            float k2 = 0.0f;
+#pragma unroll
+            for (int w = 0; w < DK / 32; ++w) k2 += sm.wsum[1][w];
+            const float xs = -expm1f(-2.0f * rate_h);
+            const float xr = p.erase ? __fmul_rn(__fmul_rn(beta, __fsub_rn(2.0f, beta)),
+                                                 __fdiv_rn(k2, static_cast<float>(DK)))
+                                     : 0.0f;
+            if (t == 0) {
+                sm.ms[0] = xs;
+                sm.mr[0] = xr;
+            } else {
+                sm.ms[0] = __fadd_rn(sm.ms[0], __fmul_rn(p.alpha, __fsub_rn(xs, sm.ms[0])));
+                sm.mr[0] = __fadd_rn(sm.mr[0], __fmul_rn(p.alpha, __fsub_rn(xr, sm.mr[0])));
+            }
+        }
+        __syncthreads();
+#pragma unroll
+        for (int r = 0; r < RPW; ++r) {
+            const float ki = sm.k[warp * RPW + r];
+#pragma unroll
+            for (int c = 0; c < CPL; ++c) x[r][c] = fmaf(ki, sm.u[lane * CPL + c], x[r][c]);
+        }
+    }
+
+    // ---- 5. write-back ------------------------------------------------------------------------
+    if (DST_PACKED) {
+        const bool refit = (p.fit_every <= 1) || ((p.w_index + h) % p.fit_every == 0);
+        if (!HEAD) {
+#pragma unroll
+            for (int r = 0; r < RPW; ++r) {
+                const int i = warp * RPW + r;
+                RowVals<CPL> xv;
+#pragma unroll
+                for (int c = 0; c < CPL; ++c) xv.v[c] = x[r][c];
+                const RowOut o = quantise_row<CPL, DV>(xv, sm.w_out[i], lane, refit, sm.fidx_in[i],
+                                                       pay + sm.off_out[i]);
+                if (lane == 0) {
+                    if (p.range != nullptr) p.range[ubase + i] = o.R;
+                    p.out_scales[gbase + i] = static_cast<uint16_t>(o.scale);
+                    p.out_fidx[gbase + i] = static_cast<uint8_t>(o.fidx);
+                }
+            }
+        } else {
+            // head unit: one width per head; scale groups = 32 key rows x one value column.
+            // Warps 2m and 2m+1 hold the two halves of row block m.
+            const int w = sm.w_out[0];
+            const int blk = warp >> 1;
+            float* mine = sm.colmax + warp * DV;
+            const float* other = sm.colmax + (warp ^ 1) * DV;
+            float R[CPL], Dc[CPL], ic[CPL];
+            int fc[CPL];
+#pragma unroll
+            for (int c = 0; c < CPL; ++c) {
+                float m = 0.0f;
+#pragma unroll
+                for (int r = 0; r < RPW; ++r) m = (w == 1) ? m + fabsf(x[r][c]) : fmaxf(m, fabsf(x[r][c]));
+                mine[lane * CPL + c] = m;
+            }
+            __syncthreads();
+#pragma unroll
+            for (int c = 0; c < CPL; ++c) {
+                const float a = mine[lane * CPL + c], o2 = other[lane * CPL + c];
+                // same combination order in both warps of the pair: even half first
+                R[c] = (w == 1) ? ((warp & 1) ? o2 + a : a + o2) : fmaxf(a, o2);
+                fc[c] = sm.fidx_in[blk * DV + lane * CPL + c];
+            }
+            uint32_t n = 0;
+            float nf = 0.0f, inv_n = 0.0f;
+            if (w >= 2) {
+                n = (1u << (w - 1)) - 1u;
+                nf = static_cast<float>(n);
+                inv_n = __frcp_rn(nf);
+            }
+            if (w >= 2 && refit) {
+                float best[CPL];
+#pragma unroll
+                for (int c = 0; c < CPL; ++c) best[c] = INFINITY;
+                float* part = sm.fit_red + warp * 4 * DV;
+                const float* opart = sm.fit_red + (warp ^ 1) * 4 * DV;
+#pragma unroll 1
+                for (int round = 0; round < 4; ++round) {
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk) {
+                        const float f = fit_factor(round * 4 + kk);
+#pragma unroll
+                        for (int c = 0; c < CPL; ++c) {
+                            const float D = cand_step(f, R[c], inv_n);
+                            const float inv = step_rcp(D);
+                            float acc = 0.0f;
+#pragma unroll
+                            for (int r = 0; r < RPW; ++r) {
+                                const float a = fabsf(x[r][c]);
+                                const float tq = fminf(__fadd_rn(__fmul_rn(a, inv), kMagic), kMagic + nf);
+                                const float e = fmaf(-__fsub_rn(tq, kMagic), D, a);
+                                acc = fmaf(e, e, acc);
+                            }
+                            part[kk * DV + lane * CPL + c] = acc;
+                        }
+                    }
+                    __syncthreads();
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk) {
+#pragma unroll
+                        for (int c = 0; c < CPL; ++c) {
+                            const float a = part[kk * DV + lane * CPL + c], o2 = opart[kk * DV + lane * CPL + c];
+                            const float tot = (warp & 1) ? o2 + a : a + o2;
+                            if (R[c] == 0.0f) {
+                                fc[c] = kNFit - 1;
+                            } else if (tot <= best[c]) {
+                                best[c] = tot;
+                                fc[c] = round * 4 + kk;
+                            }
+                        }
+                    }
+                    __syncthreads();
+                }
+            }
+#pragma unroll
+            for (int c = 0; c < CPL; ++c) {
+                if (w >= 2) {
+                    Dc[c] = (R[c] == 0.0f) ? 0.0f : cand_step(fit_factor(fc[c]), R[c], inv_n);
+                } else if (w == 1) {
+                    Dc[c] = f16_round(__fdiv_rn(R[c], 32.0f));
+                } else {
+                    Dc[c] = 0.0f;
+                }
+                ic[c] = step_rcp(Dc[c]);
+            }
+#pragma unroll
+            for (int r = 0; r < RPW; ++r) {
+                const int i = warp * RPW + r;
+                uint32_t u[CPL];
+#pragma unroll
+                for (int c = 0; c < CPL; ++c) {
+                    if (w >= 2) {
+                        const float tq = code_magic(x[r][c], ic[c], kMagic - nf, kMagic + nf);
+                        u[c] = __float_as_uint(tq) - (kMagicBits - n);
+                    } else if (w == 1) {
+                        u[c] = x[r][c] < 0.0f ? 1u : 0u;
+                    } else {
+                        u[c] = 0u;
+                    }
+                }
+                store_codes<CPL>(pay + sm.off_out[i], lane, w, u);
+            }
+            if ((warp & 1) == 0) {
+#pragma unroll
+                for (int c = 0; c < CPL; ++c) {
+                    const int g = blk * DV + lane * CPL + c;
+                    p.out_scales[gbase + g] = f16_bits(Dc[c]);
+                    p.out_fidx[gbase + g] = static_cast<uint8_t>(fc[c]);
+                }
+            }
+        }
+        __syncthreads();
+        const int nbytes = sm.off_out[DK];
+        Vec* dst = reinterpret_cast<Vec*>(p.out_payload + static_cast<size_t>(b) * p.region_bytes +
+                                          p.out_head_off[bh]);
+        const Vec* srcv = reinterpret_cast<const Vec*>(pay);
+        const int nv = nbytes / static_cast<int>(sizeof(Vec));
+        for (int i = tid; i < nv; i += 256) dst[i] = srcv[i];
+    } else if (p.dense_out != nullptr) {
+#pragma unroll
+        for (int r = 0; r < RPW; ++r) {
+            const int i = warp * RPW + r;
+            float* dst = p.dense_out + (static_cast<size_t>(bh) * DK + i) * DV + lane * CPL;
+            if (CPL == 4) {
+                *reinterpret_cast<float4*>(dst) =
+                    make_float4(x[r][0], x[r][1], x[r][CPL > 2 ? 2 : 0], x[r][CPL > 3 ? 3 : 0]);
+            } else {
+                *reinterpret_cast<float2*>(dst) = make_float2(x[r][0], x[r][1]);
+            }
+        }
+    }
+    if (stats) {
+        if (!HEAD) {
+            for (int i = tid; i < DK; i += 256) {
+                p.ema_s[ubase + i] = sm.ms[i];
+                p.ema_r[ubase + i] = sm.mr[i];
+            }
+        } else if (tid == 0) {
+            p.ema_s[ubase] = sm.ms[0];
+            p.ema_r[ubase] = sm.mr[0];
+        }
+    }
+}
+
+template <int DK, int DV, bool HEAD, bool SRC_PACKED, bool DST_PACKED>
+cudaError_t launch_step_t(const qstate_cfg& cfg, const StepParams& p, cudaStream_t stream) {
+    auto kern = step_kernel<DK, DV, HEAD, SRC_PACKED, DST_PACKED>;
+    const size_t smem = sizeof(StepSmem<DK, DV, HEAD>) +
+                        ((SRC_PACKED || DST_PACKED) ? static_cast<size_t>(DK) * DV * cfg.bmax / 8 + 32 : 0);
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    StepParams q = p;
+    q.stage_bytes = DK * DV * cfg.bmax / 8;
+    kern<<<cfg.B * cfg.H, 256, smem, stream>>>(q);
+    return cudaGetLastError();
+}
+
+template <int DK, int DV>
+cudaError_t launch_step_shape(const qstate_cfg& cfg, int src_packed, int dst_packed,
+                              const StepParams& p, cudaStream_t stream) {
+    const bool head = cfg.unit_kind == QSTATE_UNIT_HEAD;
+#define QS_CASE(HD, SP, DP)                                                            \
+    if (head == HD && (src_packed != 0) == SP && (dst_packed != 0) == DP)              \
+        return launch_step_t<DK, DV, HD, SP, DP>(cfg, p, stream);
+    QS_CASE(false, true, true)
+    QS_CASE(false, false, true)
+    QS_CASE(false, true, false)
+    QS_CASE(false, false, false)
+    if (DK % 32 == 0) {
+        QS_CASE(true, true, true)
+        QS_CASE(true, false, true)
+        QS_CASE(true, true, false)
+    }
+#undef QS_CASE
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace qs

@@ -1,0 +1,377 @@
+"""GPU parity tests: the CUDA library (through the C ABI) against the CPU oracle on identical
+seeded inputs.  Bit-exact: allocation, initial state, pack/unpack layout, log-decay codes.
+Floating point: unquantised FP32 recurrence (free-running, 1e-5), quantised write-backs in
+lockstep (the oracle's state at each write-back is handed to the GPU; codes >= 99.99%
+identical and within one step, readouts within 1e-3)."""
+import numpy as np
+import pytest
+
+import synth
+from parity import (REL_O_FP32, REL_O_QUANT, REL_STATS, compare_packed, dev, from_gpu_state,
+                    host, rel_err_vectors, set_gpu_state)
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+def small(name, **kw):
+    return synth.scaled(synth.WORKLOADS[name], **kw)
+
+
+SMALL = {
+    "tiny_kda": small("tiny_kda", T=48),
+    "kda_decode": small("kda_decode", B=3, H=4, T=12),
+    "gdn_decode": small("gdn_decode", B=3, H=5, T=10),
+    "mamba2_decode": small("mamba2_decode", B=2, H=16, T=10, group_heads=8),
+    "kda_prefill": small("kda_prefill", B=2, H=3, T=150, C=64),
+}
+
+
+def _dev_inputs(w, inp, q, s_code=None, s_lut=None):
+    d = {k: dev(v, torch) for k, v in inp.items()}
+    if s_code is not None:
+        return q.Inputs(d["q"], d["k"], d["v"], None, dev(s_code, torch), dev(s_lut, torch),
+                        d["beta"], w.T), d
+    return q.Inputs(d["q"], d["k"], d["v"], d["s"], None, None, d["beta"], w.T), d
+
+
+def _random_stats(cfg, rng, zero_group=False, null_rows=0):
+    n = cfg.B * cfg.units
+    s = np.exp(rng.uniform(np.log(1e-4), np.log(3.0), n))
+    ms = (-np.expm1(-2 * s)).astype(np.float32)
+    mr = rng.uniform(0, 0.05, n).astype(np.float32)
+    R = np.exp(rng.normal(0, 1.5, n)).astype(np.float32)
+    if zero_group:
+        R[: cfg.group_heads * cfg.dk] = 0
+    if null_rows:
+        ms[rng.choice(n, null_rows, replace=False)] = 1.0   # Gamma_hat = 0
+    return ms, mr, R
+
+
+# ------------------------------------------------------------------------------ bit-exact units
+@pytest.mark.parametrize("name", ["tiny_kda", "kda_decode", "gdn_decode", "mamba2_decode", "kda_prefill"])
+def test_alloc_bit_exact(qs, orc, name):
+    w = synth.WORKLOADS[name]
+    w = synth.scaled(w, B=min(w.B, 6))
+    cfgq, cfgo = qs.Config.from_workload(w), orc.Cfg.from_workload(w)
+    rng = np.random.default_rng(7)
+    for trial in range(4):
+        ms, mr, R = _random_stats(cfgo, rng, zero_group=(trial == 1), null_rows=7 if trial == 2 else 0)
+        if trial == 3:
+            ms[:] = ms[0]; mr[:] = mr[0]; R[:] = R[0]           # all tied
+        st = qs.Stats(dev(ms, torch), dev(mr, torch), dev(R, torch))
+        widths = torch.zeros(cfgq.B * cfgq.units, dtype=torch.uint8, device="cuda")
+        head_off = torch.zeros(cfgq.B * cfgq.H, dtype=torch.int32, device="cuda")
+        qs.qstate_alloc_bits(cfgq, st, widths, head_off)
+        qs.qstate_check()
+        wref, oref = orc.alloc(cfgo, ms, mr, R)
+        assert np.array_equal(host(widths, np.uint8), wref), (name, trial)
+        assert np.array_equal(host(head_off, np.uint32), oref), (name, trial)
+
+
+@pytest.mark.parametrize("name", ["tiny_kda", "kda_decode", "gdn_decode", "mamba2_decode"])
+def test_init_bit_exact(qs, orc, name):
+    w = synth.scaled(synth.WORKLOADS[name], B=2)
+    cfgq, cfgo = qs.Config.from_workload(w), orc.Cfg.from_workload(w)
+    a, b = qs.new_state(cfgq), qs.new_state(cfgq)
+    qs.qstate_init(cfgq, a, b)
+    qs.qstate_check()
+    ra, rb = orc.init_state(cfgo)
+    ga, gb = from_gpu_state(orc, a), from_gpu_state(orc, b)
+    for f in ("payload", "scales", "widths", "head_off", "fidx"):
+        assert np.array_equal(getattr(ga, f), getattr(ra, f)), f
+    assert np.array_equal(gb.widths, rb.widths) and np.array_equal(gb.head_off, rb.head_off)
+
+
+def _width_map(cfgo, rng, lo, hi):
+    """Random widths in [lo, hi] meeting the budget exactly, with offsets."""
+    N = cfgo.units
+    total = N * cfgo.bbar_num // cfgo.bbar_den
+    ws = []
+    for b in range(cfgo.B):
+        w = np.full(N, total // N)
+        for _ in range(4 * N):
+            i, j = rng.integers(0, N, 2)
+            if w[i] < hi and w[j] > lo:
+                w[i] += 1
+                w[j] -= 1
+        ws.append(w)
+    wv = np.stack(ws).astype(np.uint8)
+    rows = wv if cfgo.unit_kind == 0 else np.repeat(wv, cfgo.dk, axis=1)
+    row_bytes = rows.reshape(cfgo.B, cfgo.H, cfgo.dk).astype(int) * cfgo.dv // 8
+    hb = row_bytes.sum(2)
+    off = np.concatenate([np.zeros((cfgo.B, 1), int), np.cumsum(hb, 1)[:, :-1]], 1)
+    return wv.ravel(), off.astype(np.uint32).ravel()
+
+
+@pytest.mark.parametrize("name,lo,hi", [("kda_decode", 0, 16), ("tiny_kda", 0, 16),
+                                        ("gdn_decode", 2, 16), ("mamba2_decode", 1, 16)])
+def test_pack_unpack_vs_oracle(qs, orc, name, lo, hi):
+    w = synth.scaled(synth.WORKLOADS[name], B=2, bmin=lo, bmax=hi)
+    cfgq, cfgo = qs.Config.from_workload(w), orc.Cfg.from_workload(w)
+    rng = np.random.default_rng(11)
+    widths, head_off = _width_map(cfgo, rng, lo, hi)
+    S = synth.random_state(w, 3)
+    # edge rows: all zero, a single spike, tiny (FP16 subnormal steps) and huge ranges
+    S[0, 0, 0] = 0
+    S[0, 0, 1] = 0
+    S[0, 0, 1, 5] = -3.0
+    S[0, 0, 2] *= 1e-6
+    S[0, 0, 3] *= 1e3
+    ref_payload, ref_scales, ref_fidx, ref_range = orc.pack(cfgo, S, widths, head_off)
+    ref = orc.Buf(ref_payload, ref_scales, widths, head_off, ref_fidx)
+    st = qs.new_state(cfgq)
+    st.widths.copy_(dev(widths, torch))
+    st.head_off.copy_(dev(head_off, torch))
+    rng_out = torch.zeros(cfgq.B * cfgq.units, dtype=torch.float32, device="cuda")
+    qs.qstate_pack(cfgq, dev(S, torch), st, rng_out if cfgq.unit_kind == 0 else None)
+    qs.qstate_check()
+    gpu = from_gpu_state(orc, st)
+    compare_packed(orc, cfgo, gpu, ref, X=S)
+    if cfgq.unit_kind == 0:
+        assert np.array_equal(host(rng_out, np.float32), ref_range)
+    # unpack is bit-exact on both payloads
+    for buf in (ref, gpu):
+        set_gpu_state(st, buf)
+        out = torch.empty(S.shape, dtype=torch.float32, device="cuda")
+        qs.qstate_unpack(cfgq, st, out)
+        qs.qstate_check()
+        X = orc.unpack(cfgo, buf.payload, buf.scales, buf.widths, buf.head_off)
+        assert np.array_equal(host(out, np.float32), X)
+
+
+@pytest.mark.parametrize("name,g", [("kda_decode", 2), ("kda_decode", 4), ("gdn_decode", 2),
+                                    ("mamba2_decode", 1)])
+def test_quant_decay_bit_exact(qs, orc, name, g):
+    w = synth.scaled(synth.WORKLOADS[name], B=3, T=40, gate_bits=g)
+    cfgq = qs.Config.from_workload(w)
+    inp = synth.host_inputs(w)
+    s = inp["s"]
+    nchan = w.H * w.dk if w.per_row_decay else w.H
+    codes = torch.zeros(s.shape, dtype=torch.uint8, device="cuda")
+    lut = torch.zeros(nchan * 2 ** g, dtype=torch.float32, device="cuda")
+    thr = torch.zeros(nchan * (2 ** g - 1), dtype=torch.float32, device="cuda")
+    qs.qstate_quant_decay(cfgq, dev(s, torch), codes, lut, thr)
+    qs.qstate_check()
+    c_ref, l_ref, t_ref = orc.quant_decay(s, nchan, g)
+    assert np.array_equal(host(lut, np.float32).reshape(nchan, -1), l_ref)
+    assert np.array_equal(host(thr, np.float32).reshape(nchan, -1), t_ref)
+    assert np.array_equal(host(codes, np.uint8), c_ref)
+
+
+# ------------------------------------------------------------------ unquantised FP32 recurrence
+@pytest.mark.parametrize("name", ["tiny_kda", "kda_decode", "gdn_decode", "mamba2_decode", "kda_prefill"])
+def test_fp32_recurrence_free_running(qs, orc, name):
+    w = SMALL[name] if name != "tiny_kda" else synth.WORKLOADS["tiny_kda"]
+    cfgq, cfgo = qs.Config.from_workload(w, gate_bits=0), orc.Cfg.from_workload(w, gate_bits=0)
+    inp = synth.host_inputs(w)
+    X, _ = _dev_inputs(w, inp, qs)
+    S = torch.zeros((w.B, w.H, w.dk, w.dv), dtype=torch.float32, device="cuda")
+    o = torch.zeros((w.B, w.T, w.H, w.dv), dtype=torch.float32, device="cuda")
+    qs.qstate_scan_fp32(cfgq, S, X, 0, w.T, o)
+    qs.qstate_check()
+    og = host(o, np.float32)
+    worst32 = worst64 = 0.0
+    for b in range(w.B):
+        for h in range(w.H):
+            args = orc.expand_inputs(cfgo, inp, b, h)
+            o32, _ = orc.recur(np.zeros((w.dk, w.dv)), *args, dtype=np.float32)
+            o64, _ = orc.recur(np.zeros((w.dk, w.dv)), *args, dtype=np.float64)
+            worst32 = max(worst32, rel_err_vectors(og[b, :, h], o32))
+            worst64 = max(worst64, rel_err_vectors(og[b, :, h], o64))
+    print(f"{name}: max rel readout error vs FP32 oracle {worst32:.2e}, vs FP64 {worst64:.2e}")
+    assert worst32 <= REL_O_FP32
+    assert worst64 <= REL_O_FP32
+
+
+# --------------------------------------------------------------- quantised write-backs, lockstep
+def _lockstep(qs, orc, w, fit_every=1, log_decay=False, sample_b=None, max_wb=None):
+    """Run the oracle free; before every write-back copy its state into the GPU, run one
+    qstate_step and compare the GPU's write-back with the oracle's.  With sample_b, the GPU
+    runs the full batch and only those batch elements are injected and compared (the oracle
+    runs a B=1 configuration per sampled element)."""
+    cfgq = qs.Config.from_workload(w, fit_every=fit_every)
+    cfgo_full = orc.Cfg.from_workload(w, fit_every=fit_every)
+    inp = synth.host_inputs(w)
+    s_code = s_lut = None
+    if log_decay:
+        nchan = w.H * w.dk if w.per_row_decay else w.H
+        s_code, s_lut, _ = orc.quant_decay(inp["s"], nchan, w.gate_bits)
+    X, _ = _dev_inputs(w, inp, qs, s_code, s_lut)
+    bs = list(range(w.B)) if sample_b is None else list(sample_b)
+    one = sample_b is not None
+    cfgo = orc.Cfg.from_workload(synth.scaled(w, B=1), fit_every=fit_every) if one else cfgo_full
+    sub = (lambda a, b: a[b:b + 1]) if one else (lambda a, b: a)
+    orc_inp = {b: {k: sub(v, b) for k, v in inp.items()} for b in (bs if one else [0])}
+    orc_code = {b: (sub(s_code, b) if s_code is not None else None) for b in (bs if one else [0])}
+    # oracle states per (sampled) batch element
+    states = {}
+    for key in (bs if one else [0]):
+        src, dst = orc.init_state(cfgo)
+        z = lambda: np.zeros(cfgo.B * cfgo.units, np.float32)
+        states[key] = dict(src=src, dst=dst, ms=z(), mr=z(), R=z(),
+                           o=np.zeros((cfgo.B, w.T, w.H, w.dv), np.float32))
+    A, Bst = qs.new_state(cfgq), qs.new_state(cfgq)
+    qs.qstate_init(cfgq, A, Bst)
+    gst = qs.new_stats(cfgq)
+    o = torch.zeros((w.B, w.T, w.H, w.dv), dtype=torch.float32, device="cuda")
+    region, units, groups = cfgo.region_bytes, cfgo.units, cfgo.n_scale_groups
+    report = []
+    nwb = 0
+    for wi, t0 in enumerate(range(0, w.T, w.C)):
+        if max_wb is not None and wi >= max_wb:
+            break
+        t1 = min(w.T, t0 + w.C)
+        gsrc, gdst = (A, Bst) if wi % 2 == 0 else (Bst, A)
+        # inject the oracle's state (before this write-back) into the GPU
+        for key, S in states.items():
+            bsel = key if one else None
+            kw = dict(b=key, region=region, units=units, groups=groups, H=w.H) if one else {}
+            set_gpu_state(gsrc, S["src"], **kw)
+            dst_meta = S["dst"].copy()
+            set_gpu_state(gdst, dst_meta, **kw)
+            for t, a in zip((gst.ema_s, gst.ema_r, gst.range), (S["ms"], S["mr"], S["R"])):
+                if one:
+                    t[key * units:(key + 1) * units].copy_(torch.from_numpy(a).cuda())
+                else:
+                    t.copy_(torch.from_numpy(a).cuda())
+        qs.qstate_step(cfgq, gsrc, gdst, X, t0, t1, wi, o, gst)
+        qs.qstate_check()
+        g_out = from_gpu_state(orc, gdst)
+        g_next = from_gpu_state(orc, gsrc)
+        g_ms, g_mr, g_R = (host(t, np.float32) for t in (gst.ema_s, gst.ema_r, gst.range))
+        og = host(o, np.float32)
+        for key, S in states.items():
+            xo = orc.step(cfgo, S["src"], S["dst"], orc_inp[key], t0, t1, wi, S["o"], S["ms"], S["mr"],
+                          S["R"], orc_code[key], s_lut, want_x=True)
+            sl = (slice(key, key + 1) if one else slice(None))
+            # readouts of this interval
+            e_o = rel_err_vectors(og[sl, t0:t1], S["o"][:, t0:t1])
+            assert e_o <= REL_O_QUANT, (wi, key, e_o)
+            # packed state
+            if one:
+                gb = orc.Buf(g_out.payload[key * region:(key + 1) * region],
+                             g_out.scales[key * groups:(key + 1) * groups],
+                             g_out.widths[key * units:(key + 1) * units],
+                             g_out.head_off[key * w.H:(key + 1) * w.H],
+                             g_out.fidx[key * groups:(key + 1) * groups])
+            else:
+                gb = g_out
+            st = compare_packed(orc, cfgo, gb, S["dst"], X=xo)
+            # statistics
+            us = slice(key * units, (key + 1) * units) if one else slice(None)
+            for a, r in ((g_ms[us], S["ms"]), (g_mr[us], S["mr"])):
+                assert np.allclose(a, r, rtol=REL_STATS, atol=1e-30), wi
+            if cfgo.unit_kind == 0:
+                assert np.allclose(g_R[us], S["R"], rtol=REL_STATS, atol=0), wi
+            report.append(dict(wb=wi, b=key, rel_o=e_o, **st))
+            # next widths: the oracle's allocation of its own statistics; the GPU's allocation
+            # of the same statistics must agree bit for bit (checked through qstate_alloc_bits)
+            wn, on = orc.alloc(cfgo, S["ms"], S["mr"], S["R"])
+            sts = qs.Stats(dev(S["ms"], torch), dev(S["mr"], torch), dev(S["R"], torch))
+            cq = qs.Config.from_workload(synth.scaled(w, B=cfgo.B), fit_every=fit_every)
+            wt = torch.zeros(cfgo.B * units, dtype=torch.uint8, device="cuda")
+            ot = torch.zeros(cfgo.B * w.H, dtype=torch.int32, device="cuda")
+            qs.qstate_alloc_bits(cq, sts, wt, ot)
+            assert np.array_equal(host(wt, np.uint8), wn) and np.array_equal(host(ot, np.uint32), on)
+            # the GPU's own next widths (from its own statistics) agree almost everywhere
+            agree = np.mean(g_next.widths[us] == wn)
+            assert agree >= 0.99, (wi, key, agree)
+            S["src"].widths[:], S["src"].head_off[:] = wn, on
+            S["src"], S["dst"] = S["dst"], S["src"]
+        nwb += 1
+    return report
+
+
+@pytest.mark.parametrize("name", ["tiny_kda", "kda_decode", "gdn_decode", "mamba2_decode", "kda_prefill"])
+def test_quantised_lockstep(qs, orc, name):
+    w = SMALL[name]
+    rep = _lockstep(qs, orc, w, log_decay=(w.gate_bits > 0))
+    worst = max(r["rel_o"] for r in rep)
+    agree = min(r["code_agree"] for r in rep)
+    ties = sum(r["fidx_diff"] for r in rep)
+    print(f"{name}: {len(rep)} write-backs, worst rel readout {worst:.2e}, min code agreement "
+          f"{agree:.6f}, near-tie factor differences {ties}")
+
+
+def test_quantised_lockstep_fit_every(qs, orc):
+    w = small("kda_decode", B=2, H=4, T=10, gate_bits=0)
+    _lockstep(qs, orc, w, fit_every=4)
+
+
+def test_quantised_lockstep_ragged_chunks(qs, orc):
+    w = small("kda_prefill", B=1, H=2, T=37, C=16)
+    _lockstep(qs, orc, w)
+
+
+@pytest.mark.parametrize("name,T,sample", [("kda_decode", 3, (0, 131, 255)),
+                                           ("gdn_decode", 3, (0, 63)),
+                                           ("mamba2_decode", 2, (5, 127))])
+def test_full_size_sampled_lockstep(qs, orc, name, T, sample):
+    """Full batch and heads of the benchmark workloads, in the launch configuration the
+    benchmark times; sampled batch elements are compared write-back by write-back."""
+    w = synth.scaled(synth.WORKLOADS[name], T=T)
+    _lockstep(qs, orc, w, log_decay=(w.gate_bits > 0), sample_b=sample)
+
+
+# ---------------------------------------------------------------------------------- edge cases
+def test_inconsistent_layout_is_reported(qs, orc):
+    w = small("kda_decode", B=2, H=2, T=2, gate_bits=0)
+    cfgq = qs.Config.from_workload(w)
+    inp = synth.host_inputs(w)
+    X, _ = _dev_inputs(w, inp, qs)
+    A, Bst = qs.new_state(cfgq), qs.new_state(cfgq)
+    qs.qstate_init(cfgq, A, Bst)
+    Bst.widths[5] = 17                      # caught by the kernel's own layout check
+    o = torch.zeros((w.B, w.T, w.H, w.dv), dtype=torch.float32, device="cuda")
+    qs.qstate_step(cfgq, A, Bst, X, 0, 1, 0, o, qs.new_stats(cfgq))
+    with pytest.raises(qs.QstateError) as e:
+        qs.qstate_check()
+    assert e.value.code == qs.QSTATE_EDEVICE
+    qs.qstate_check()                       # cleared
+
+
+def test_host_side_argument_errors(qs):
+    cfg = qs.Config.from_workload(small("kda_decode", B=1, H=2, T=2))
+    A, Bst = qs.new_state(cfg), qs.new_state(cfg)
+    o = torch.zeros((1, 2, 2, 128), device="cuda")
+    z = torch.zeros((1, 2, 2, 128), device="cuda")
+    X = qs.Inputs(z, z, z, None, None, None, torch.zeros((1, 2, 2), device="cuda"), 2)
+    with pytest.raises(qs.QstateError):
+        qs.qstate_step(cfg, A, Bst, X, 0, 1, 0, o, qs.new_stats(cfg))   # no decay rates
+    X.s = torch.ones((1, 2, 2, 128), device="cuda")
+    with pytest.raises(qs.QstateError):
+        qs.qstate_step(cfg, A, Bst, X, 0, 2, 0, o, qs.new_stats(cfg))   # 2 tokens > C = 1
+    bad = qs.Config.from_workload(small("kda_decode", B=1, H=2, T=2), bmin=5)
+    with pytest.raises(qs.QstateError) as e:
+        qs.qstate_init(bad, A, Bst)
+    assert e.value.code == qs.QSTATE_EBUDGET
+
+
+def test_scan_equals_repeated_steps(qs, orc):
+    """qstate_scan = the sequence of qstate_step calls, bit for bit."""
+    w = small("kda_prefill", B=2, H=2, T=40, C=16)
+    cfgq = qs.Config.from_workload(w)
+    inp = synth.host_inputs(w)
+    X, _ = _dev_inputs(w, inp, qs)
+    outs = []
+    for mode in ("scan", "steps"):
+        A, Bst = qs.new_state(cfgq), qs.new_state(cfgq)
+        qs.qstate_init(cfgq, A, Bst)
+        st = qs.new_stats(cfgq)
+        o = torch.zeros((w.B, w.T, w.H, w.dv), dtype=torch.float32, device="cuda")
+        if mode == "scan":
+            pong = qs.qstate_scan(cfgq, A, Bst, X, 0, w.T, 0, o, st)
+            fin = Bst if pong else A
+        else:
+            src, dst = A, Bst
+            for wi, t0 in enumerate(range(0, w.T, w.C)):
+                qs.qstate_step(cfgq, src, dst, X, t0, min(w.T, t0 + w.C), wi, o, st)
+                src, dst = dst, src
+            fin = src
+        qs.qstate_check()
+        outs.append((host(o, np.float32), from_gpu_state(orc, fin)))
+    assert np.array_equal(outs[0][0], outs[1][0])
+    for f in ("payload", "scales", "widths", "head_off", "fidx"):
+        assert np.array_equal(getattr(outs[0][1], f), getattr(outs[1][1], f))
