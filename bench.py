@@ -1,0 +1,379 @@
+"""Benchmark of the quantised-state recurrence on GB300.
+
+A step is one pass of the whole hot path over one batch of the KDA decode workload
+(B = 256, H = 32, dk = dv = 128, T = 1024 tokens, per-token write-back, 4-bit mean payload,
+widths 0..8, log-quantised decay rates with 2 bits): the log-uniform decay quantiser over the
+batch's rates, then T write-backs, each the fused write-back kernel followed by the bit
+allocation for the next one.  Inputs (17 GB) are resident in HBM when the timed region starts
+and exceed L2, so no flush is needed.  Prints one JSON line.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference] [--fit-every F]
+
+Under torchrun each rank runs the same per-GPU batch (batch elements are independent: weak
+scaling, no collective); the reported value is the sum over ranks divided by the slowest rank.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+WORKLOAD = "kda_decode"
+PEAK_FALLBACK_GBS = 6800.0
+
+
+def algorithmic_bytes(w, fit_every=1):
+    """Bytes the method must move per write-back launch (the fused kernel) and per allocation
+    launch, itemised per head for the row unit with log-coded rates:
+      payload read + write        2 dk dv bbar / 8
+      FP16 scales read + write    2 * 2 dk
+      widths read (in + out)      2 dk
+      fitted-factor index r + w   2 dk
+      head offsets (in + out)     8
+      EMA statistics r + w        2 * 2 * 4 dk
+      row range write             4 dk
+      q, k, v                     4 (2 dk + dv)
+      rate codes + beta           dk + 4
+      readout o                   4 dv
+    Allocation per batch element: EMA + range read 12 per row, widths 1 per row, offsets 4 H."""
+    dk, dv = w.dk, w.dv
+    per_head = (2 * dk * dv * w.bbar // 8 + 4 * dk + 2 * dk + 2 * dk + 8 + 16 * dk + 4 * dk +
+                4 * (2 * dk + dv) + (dk if w.gate_bits else 4 * dk) + 4 + 4 * dv)
+    writeback = per_head * w.B * w.H
+    alloc = w.B * (w.H * dk * 13 + 4 * w.H)
+    return writeback, alloc, per_head
+
+
+def kernel_sha():
+    """Hash of the sources of the fused write-back kernel (ties an ncu traffic figure to the
+    kernel it was taken on)."""
+    h = hashlib.sha256()
+    for f in ("qs_step_impl.cuh", "qs_common.cuh", "qs_internal.h"):
+        with open(os.path.join(ROOT, "paper_2609_30950_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(sha):
+    """DRAM bytes per write-back launch from the committed ncu summary, if it was taken on
+    the current kernel sources; else None."""
+    path = os.path.join(ROOT, "profiles", "writeback_kda_decode.md")
+    if not os.path.exists(path):
+        return None
+    vals = {}
+    for line in open(path):
+        if ":" in line and line.strip().startswith("- "):
+            k, v = line.strip()[2:].split(":", 1)
+            vals[k.strip()] = v.strip()
+    if vals.get("kernel_sha") != sha:
+        return None
+    try:
+        return float(vals["dram_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return PEAK_FALLBACK_GBS, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+
+    def __init__(self, gpu_index=0):
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{gpu_index}.csv")
+        os.makedirs(os.path.dirname(self.path), exist_ok=True)
+        self.idx = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        try:
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.idx}", f"--query-gpu={q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.fh, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.fh.close()
+
+    def summary(self):
+        try:
+            rows = [r.split(",") for r in open(self.path).read().strip().splitlines() if r.strip()]
+        except Exception:
+            return None
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].strip().replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].strip().replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = set()
+        for r in rows:
+            for n, v in zip(names, r[5:9]):
+                if v.strip().lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons),
+                "samples": len(rows)}
+
+
+def cpu_baseline(w, budget_s=12.0):
+    """The oracle as it stands, single-threaded, on a bounded sample of the workload: the
+    log-decay quantiser over the sample's rates, then per token one write-back of every head
+    of the sampled batch elements and the allocation.  Returns tokens/s and the sample."""
+    import numpy as np
+    from oracle import oracle as orc
+    nb, nt = 4, 64
+    sub = synth.scaled(w, B=nb)
+    cfg = orc.Cfg.from_workload(sub)
+    t_start = time.perf_counter()
+    inp = synth.host_inputs(sub, t_range=(0, nt))
+    gen_s = time.perf_counter() - t_start
+    t0 = time.perf_counter()
+    nchan = w.H * w.dk
+    codes, lut, _ = orc.quant_decay(inp["s"], nchan, w.gate_bits)
+    src, dst = orc.init_state(cfg)
+    o = np.zeros((nb, nt, w.H, w.dv), np.float32)
+    ms, mr, R = (np.zeros(cfg.units * nb, np.float32) for _ in range(3))
+    tokens = 0
+    for t in range(nt):
+        orc.step(cfg, src, dst, inp, t, t + 1, t, o, ms, mr, R, codes, lut)
+        src.widths[:], src.head_off[:] = orc.alloc(cfg, ms, mr, R)
+        src, dst = dst, src
+        tokens += nb
+        if time.perf_counter() - t0 > budget_s:
+            break
+    el = time.perf_counter() - t0
+    return tokens / el, dict(cores=1, sample=f"{nb} batch elements x {tokens // nb} tokens x "
+                                             f"{w.H} heads, single thread (input synthesis "
+                                             f"{gen_s:.1f}s excluded)",
+                             seconds=el)
+
+
+def run_reference(args, w):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    vals = []
+    for i in range(args.warmup + args.steps):
+        v, info = cpu_baseline(w, budget_s=max(3.0, 40.0 / max(1, args.steps + args.warmup)))
+        if i >= args.warmup:
+            vals.append(v)
+    value = statistics.median(vals)
+    line = {"metric": "quantised-state decode tokens/s (1 layer)", "value": value,
+            "unit": "tokens/s", "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1000.0 * w.B * w.T / value, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "impl": "reference",
+            "config": config_of(w, args),
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": info["cores"],
+                             "kind": "oracle", "sample": info["sample"]},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+def config_of(w, args):
+    return {"workload": w.name, "B": w.B, "H": w.H, "dk": w.dk, "dv": w.dv, "T": w.T, "C": w.C,
+            "bbar": w.bbar, "widths": [w.bmin, w.bmax], "gate_bits": w.gate_bits,
+            "fit_every": args.fit_every, "global_batch": w.B * args.gpus, "seq_len": w.T,
+            "parallelism": f"dp{args.gpus}", "l2": "inputs 17 GB > 129 MB L2: no flush"}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--fit-every", type=int, default=1)
+    ap.add_argument("--T", type=int, default=None, help="tokens per step (default: workload T)")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    w = synth.WORKLOADS[WORKLOAD]
+    if args.T:
+        w = synth.scaled(w, T=args.T)
+    if args.impl == "reference":
+        return run_reference(args, w)
+
+    import torch
+    import torch.distributed as dist
+    import paper_2609_30950_gb300 as q
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    q.load(build_if_missing=True)
+
+    cfg = q.Config.from_workload(w, fit_every=args.fit_every)
+    x = synth.device_inputs(w, device=dev, seed_offset=rank)
+    nchan = w.H * w.dk
+    L = 1 << w.gate_bits
+    codes = torch.empty(x["s"].shape, dtype=torch.uint8, device=dev)
+    lut = torch.empty(nchan * L, dtype=torch.float32, device=dev)
+    thr = torch.empty(nchan * (L - 1), dtype=torch.float32, device=dev)
+    o = torch.empty((w.B, w.T, w.H, w.dv), dtype=torch.float32, device=dev)
+    A, Bst = q.new_state(cfg, dev), q.new_state(cfg, dev)
+    st = q.new_stats(cfg, dev)
+    X = q.Inputs(x["q"], x["k"], x["v"], None, codes, lut, x["beta"], w.T)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        q.qstate_quant_decay(cfg, x["s"], codes, lut, thr, stream)
+        q.qstate_init(cfg, A, Bst, stream)
+        q.qstate_scan(cfg, A, Bst, X, 0, w.T, 0, o, st, stream)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    for _ in range(args.warmup):
+        step()
+    q.qstate_check(stream)
+    barrier()
+
+    # timed region: K steps; events split each step into the decay quantiser and the scan
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+           torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    with ClockSampler(local) as clk:
+        barrier()
+        t0 = time.perf_counter()
+        start = torch.cuda.Event(enable_timing=True)
+        end = torch.cuda.Event(enable_timing=True)
+        start.record(stream)
+        for e0, e1, e2 in ev:
+            e0.record(stream)
+            q.qstate_quant_decay(cfg, x["s"], codes, lut, thr, stream)
+            q.qstate_init(cfg, A, Bst, stream)
+            e1.record(stream)
+            q.qstate_scan(cfg, A, Bst, X, 0, w.T, 0, o, st, stream)
+            e2.record(stream)
+        end.record(stream)
+        barrier()
+        wall = time.perf_counter() - t0
+    q.qstate_check(stream)
+    ms_total = start.elapsed_time(end)
+    if world > 1:
+        t = torch.tensor([ms_total], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_total = float(t.item())
+    ms_step = ms_total / args.steps
+    tokens_step = w.B * w.T
+    value = tokens_step * world / (ms_step / 1000.0)
+    scan_ms = statistics.median(e1.elapsed_time(e2) for _, e1, e2 in ev)
+    decay_ms = statistics.median(e0.elapsed_time(e1) for e0, e1, _ in ev)
+    per_wb_ms = scan_ms / w.T        # write-back kernel + allocation kernel per token
+
+    wb_bytes, alloc_bytes, per_head = algorithmic_bytes(w, args.fit_every)
+    peak, peak_kind = peaks()
+    achieved = (wb_bytes + alloc_bytes) / (per_wb_ms / 1000.0) / 1e9
+    sha = kernel_sha()
+    traffic = recorded_traffic(sha)
+
+    # end to end through the public API: pinned host inputs -> device, the step, o -> host
+    e2e = None
+    if not args.no_e2e:
+        names = ["q", "k", "v", "s", "beta"]
+        host_in = {n: torch.empty(x[n].shape, dtype=x[n].dtype, pin_memory=True) for n in names}
+        for n in names:
+            host_in[n].copy_(x[n])
+        host_o = torch.empty(o.shape, dtype=o.dtype, pin_memory=True)
+        h2d = sum(t.numel() * t.element_size() for t in host_in.values())
+        d2h = host_o.numel() * host_o.element_size()
+
+        def e2e_step():
+            for n in names:
+                x[n].copy_(host_in[n], non_blocking=True)
+            step()
+            host_o.copy_(o, non_blocking=True)
+
+        e2e_step()
+        barrier()
+        k2 = max(1, min(args.steps, 3))
+        s0 = torch.cuda.Event(enable_timing=True)
+        s1 = torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        for _ in range(k2):
+            e2e_step()
+        s1.record(stream)
+        barrier()
+        e_ms = s0.elapsed_time(s1) / k2
+        if world > 1:
+            t = torch.tensor([e_ms], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e_ms = float(t.item())
+        e2e = {"value": tokens_step * world / (e_ms / 1000.0), "unit": "tokens/s",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e_ms}
+        q.qstate_check(stream)
+
+    launches_per_step = 4 + 2 + 2 * w.T   # decay (4), init (alloc + pack), T x (write-back + alloc)
+    clocks = clk.summary()
+    if rank != 0:
+        if world > 1:
+            dist.barrier()
+            dist.destroy_process_group()
+        return
+    cpu = None
+    if not args.no_cpu:
+        v, info = cpu_baseline(w)
+        cpu = {"value": v, "unit": "tokens/s", "cores": info["cores"], "kind": "oracle",
+               "sample": info["sample"]}
+    line = {
+        "metric": "quantised-state decode tokens/s (1 layer)", "value": value, "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic", "config": config_of(w, args),
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic, "peak_source": peak_kind,
+                     "kernel": "write-back + allocation per token",
+                     "algorithmic_bytes_per_launch": wb_bytes + alloc_bytes,
+                     "kernel_sha": sha},
+        "breakdown": {"decay_quantiser_ms": decay_ms, "scan_ms": scan_ms,
+                      "per_writeback_us": per_wb_ms * 1000.0, "wall_s": wall,
+                      "bits_per_element": q.bits_per_element(cfg),
+                      "pct_of_8TBps": 100.0 * achieved / 8000.0},
+        "e2e": e2e, "gpu_launches": launches_per_step * args.steps, "clocks": clocks,
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line))
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -96,23 +96,26 @@ __global__ void __launch_bounds__(kThreads) alloc_kernel(const AllocParams p) {
     long long* key = reinterpret_cast<long long*>(smem);
     const int gsz = p.group_heads * p.dk;
     const int ngroups = p.unit_row ? N / gsz : 0;
-    float* gmean = reinterpret_cast<float*>(key + N);
+    float* Rs = reinterpret_cast<float*>(key + N);                   // row unit: ranges
+    float* gmean = Rs + (p.unit_row ? N : 0);
     long long* redl = reinterpret_cast<long long*>(gmean + ((ngroups + 3) & ~3));
     int* redi = reinterpret_cast<int*>(redl + 32);
     uint8_t* wv = reinterpret_cast<uint8_t*>(redi + 72);
     const int tid = threadIdx.x;
     const size_t base = static_cast<size_t>(blockIdx.x) * N;
 
-    // 1. mean R^2 of each output-normalisation group, summed in row order (row unit)
-    if (!p.uniform)
+    // 1. mean R^2 of each output-normalisation group, summed in row order (row unit); the
+    //    ranges are staged in shared memory first so the sequential sums read on-chip data
+    if (!p.uniform && p.unit_row) {
+        for (int u = tid; u < N; u += kThreads) Rs[u] = p.range[base + u];
+        __syncthreads();
         for (int g = tid; g < ngroups; g += kThreads) {
             float acc = 0.0f;
-            for (int r = g * gsz; r < (g + 1) * gsz; ++r) {
-                const float R = p.range[base + r];
-                acc = __fadd_rn(acc, __fmul_rn(R, R));
-            }
+#pragma unroll 8
+            for (int r = g * gsz; r < (g + 1) * gsz; ++r) acc = __fadd_rn(acc, __fmul_rn(Rs[r], Rs[r]));
             gmean[g] = __fdiv_rn(acc, static_cast<float>(gsz));
         }
+    }
     __syncthreads();
 
     // 2. weights (Eq. 3) -> integer keys
@@ -127,7 +130,7 @@ __global__ void __launch_bounds__(kThreads) alloc_kernel(const AllocParams p) {
             float rt2 = 1.0f;
             if (p.unit_row) {
                 const float m = gmean[u / gsz];
-                const float R = p.range[base + u];
+                const float R = Rs[u];
                 if (m > 0.0f) rt2 = __fdiv_rn(__fmul_rn(R, R), m);
             }
             c = __fmul_rn(G, rt2);
@@ -212,8 +215,8 @@ __global__ void __launch_bounds__(kThreads) alloc_kernel(const AllocParams p) {
 
 cudaError_t launch_alloc(const AllocParams& p, cudaStream_t stream) {
     const int ngroups = p.unit_row ? p.units / (p.group_heads * p.dk) : 0;
-    const size_t smem = static_cast<size_t>(p.units) * 8 + ((ngroups + 3) & ~3) * 4 + 32 * 8 +
-                        72 * 4 + p.units + 16;
+    const size_t smem = static_cast<size_t>(p.units) * 8 + (p.unit_row ? p.units * 4 : 0) +
+                        ((ngroups + 3) & ~3) * 4 + 32 * 8 + 72 * 4 + p.units + 16;
     cudaError_t e = cudaFuncSetAttribute(alloc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;

@@ -11,6 +11,9 @@ namespace qs {
 cudaError_t launch_step_128x128(const qstate_cfg&, int, int, const StepParams&, cudaStream_t);
 cudaError_t launch_step_128x64(const qstate_cfg&, int, int, const StepParams&, cudaStream_t);
 cudaError_t launch_step_64x64(const qstate_cfg&, int, int, const StepParams&, cudaStream_t);
+cudaError_t launch_wb_row_128x128(const qstate_cfg&, const StepParams&, cudaStream_t);
+cudaError_t launch_wb_row_128x64(const qstate_cfg&, const StepParams&, cudaStream_t);
+cudaError_t launch_wb_row_64x64(const qstate_cfg&, const StepParams&, cudaStream_t);
 }  // namespace qs
 
 using namespace qs;
@@ -87,6 +90,7 @@ int validate(const qstate_cfg* c) {
     if (N * c->bmin > total || N * c->bmax < total)
         return fail(QSTATE_EBUDGET, "budget %lld bits per element sum outside [%lld, %lld]", total,
                     N * c->bmin, N * c->bmax);
+    if (N > 16384) return fail(QSTATE_EINVAL, "at most 16384 allocation units per batch element");
     if (c->C < 1) return fail(QSTATE_EINVAL, "C must be >= 1");
     if (c->fit_every < 1) return fail(QSTATE_EINVAL, "fit_every must be >= 1");
     if (!(c->ema_span > 0.0f)) return fail(QSTATE_EINVAL, "ema_span must be > 0");
@@ -108,6 +112,31 @@ cudaError_t launch_step_any(const qstate_cfg& c, int src_packed, int dst_packed,
     if (c.dk == 128 && c.dv == 128) return launch_step_128x128(c, src_packed, dst_packed, p, st);
     if (c.dk == 128 && c.dv == 64) return launch_step_128x64(c, src_packed, dst_packed, p, st);
     return launch_step_64x64(c, src_packed, dst_packed, p, st);
+}
+
+bool aligned16(const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; }
+
+// The persistent row-unit write-back kernel copies its inputs with 16-byte cp.async and needs
+// every per-head array 16-byte aligned; otherwise the one-head-per-CTA kernel runs.
+bool wb_row_eligible(const qstate_cfg& c, const StepParams& p) {
+    if (c.unit_kind != QSTATE_UNIT_ROW) return false;
+    const void* ptrs[] = {p.in_payload, p.in_scales, p.in_widths, p.in_fidx, p.out_payload,
+                          p.out_widths, p.q, p.k, p.v, p.ema_s, p.ema_r,
+                          p.s_code ? static_cast<const void*>(p.s_code) : static_cast<const void*>(p.s)};
+    for (const void* q : ptrs)
+        if (q && !aligned16(q)) return false;
+    if (!p.in_fidx) return false;
+    if (p.decay_row && p.s_code == nullptr && p.s == nullptr) return false;
+    return true;
+}
+
+cudaError_t launch_writeback(const qstate_cfg& c, const StepParams& p, cudaStream_t st) {
+    if (wb_row_eligible(c, p)) {
+        if (c.dk == 128 && c.dv == 128) return launch_wb_row_128x128(c, p, st);
+        if (c.dk == 128 && c.dv == 64) return launch_wb_row_128x64(c, p, st);
+        return launch_wb_row_64x64(c, p, st);
+    }
+    return launch_step_any(c, 1, 1, p, st);
 }
 
 StepParams base_params(const qstate_cfg* c, int* status) {
@@ -336,7 +365,7 @@ int qstate_step(const qstate_cfg* cfg, qstate_buf* in, qstate_buf* out, const qs
     p.ema_s = stats->ema_s;
     p.ema_r = stats->ema_r;
     p.range = stats->range;
-    e = launch_step_any(*cfg, 1, 1, p, st);
+    e = launch_writeback(*cfg, p, st);
     if (e != cudaSuccess) return cuda_fail(e, "write-back kernel");
     return run_alloc(cfg, stats->ema_s, stats->ema_r, stats->range, 0, in->widths, in->head_off,
                      status, st);

@@ -4,16 +4,19 @@
 // l owns value columns [l*CPL, (l+1)*CPL) of each of them, so one row is handled by one warp
 // and its bit width is warp-uniform.  The head's FP32 state lives in registers for the whole
 // write-back interval:
-//   1. metadata (widths -> row offsets by prefix sums, Sec. 3 "Prefix sums of widths give row
-//      offsets"), layout check;
+//   1. metadata: widths -> row byte offsets by prefix sums (Sec. 3, "Prefix sums of widths give
+//      row offsets"), layout check, per-row dequantisation constants, shared tables;
 //   2. the head's packed rows are staged in shared memory with 16-byte (dv = 128) or 8-byte
 //      (dv = 64) vector loads;
-//   3. unpack + dequantise (Sec. 3 levels);
+//   3. unpack + dequantise (Sec. 3 levels), branch-free: x = (float(u) - A) S + Bc per row;
 //   4. per token (Eq. 1): decay, fused reductions p = (beta k)^T S', r = q^T S' (per-lane
 //      partials over the warp's rows, then across warps in shared memory), delta update,
 //      readout o = S^T q = r + u (k . q) before quantisation (Sec. 2), EMA statistics (Sec. 3);
-//   5. range, fitted FP16 scale (16 candidates, Sec. 3), codes, repack to shared memory and a
-//      vector store of the head's new region.
+//   5. write-back (Sec. 3, "Levels and storage"): row ranges by warp reductions; the scalar
+//      per-row work (16 candidate FP16 steps and their reciprocals) row-parallel, one thread
+//      per row, into a shared table; then per row the squared-error search over the candidates,
+//      codes, and the row's bits OR-ed into a zeroed shared staging row; finally one vector
+//      store of the head's new region and coalesced stores of scales / factors / ranges.
 // The same template serves pack (dense -> packed, no tokens), unpack (packed -> dense) and the
 // unquantised reference path (dense -> dense).
 #pragma once
@@ -28,17 +31,25 @@ template <int DK, int DV, bool HEAD>
 struct alignas(16) StepSmem {
     static constexpr int NW = 8;
     static constexpr int NSG = HEAD ? (DK / 32) * DV : DK;
+    float cand[HEAD ? 1 : DK][kNFit][2];  // row unit: (Delta_k, 1/Delta_k) of the refit rows
     float k[DK], q[DK], d[DK];
     float v[DV], u[DV];
     float red[2][NW][DV];                 // p and r partials per warp
     float scale_in[NSG];                  // source steps / means (float)
     float ms[DK], mr[DK];                 // EMA statistics (head unit uses [0])
+    float deqA[DK], deqS[DK], deqB[DK];   // row unit dequantisation constants
+    float rowR[DK], rowM[DK], rowD[DK], rowInv[DK];
     float fit_red[HEAD ? NW * 4 * DV : 1];// head unit: partial SSEs, 4 candidates per round
     float colmax[HEAD ? NW * DV : 1];     // head unit: per-warp column maxima / sums
+    float fitf[kNFit];                    // f_k = (5 + k) / 20
+    float inv_n[17];                      // 1 / (2^(w-1) - 1), w = 2..16
     float wsum[2][NW];                    // per-warp partial k.q and |k|^2
     int off_in[DK + 1], off_out[DK + 1];  // row byte offsets inside the head (+ total)
+    uint16_t out_scale[NSG];
+    uint8_t out_fidx[NSG];
     uint8_t w_in[DK], w_out[DK];
     uint8_t fidx_in[NSG];
+    uint8_t mode[DK];                     // row unit: 1 = search the 16 candidates
     int flag;
 };
 
@@ -60,88 +71,21 @@ __device__ __forceinline__ float reduce16(float (&v)[16], int lane) {
     return v[0] + __shfl_xor_sync(kFull, v[0], 1);
 }
 
+// OR a lane's CPL codes (w bits each, CPL*w <= 64) into a zeroed shared row at bit
+// lane*CPL*w.  `words` is the row's first 32-bit word.
 template <int CPL>
-struct RowVals {
-    float v[CPL];
-};
-struct RowOut {
-    float R;
-    unsigned scale;
-    int fidx;
-};
-
-// Row unit write-back of one row (Sec. 3, "Levels and storage"): range R = max |x|, fitted
-// FP16 step (16 candidates, smallest squared error, ties to the larger factor) or 1-bit mean,
-// codes, and the row's bytes written to `row` (shared memory).  Called by all 32 lanes.
-template <int CPL, int DV>
-__device__ __noinline__ RowOut quantise_row(RowVals<CPL> xv, int w, int lane, bool refit,
-                                            int fidx_in, uint8_t* row) {
-    float amax = 0.0f;
+__device__ __forceinline__ void or_codes(uint32_t* words, int lane, int w, const uint32_t (&u)[CPL]) {
+    uint64_t chunk = 0;
 #pragma unroll
-    for (int c = 0; c < CPL; ++c) amax = fmaxf(amax, fabsf(xv.v[c]));
-    RowOut out;
-    out.R = warp_absmax(amax);
-    out.scale = 0;
-    out.fidx = fidx_in;
-    uint32_t u[CPL];
-    if (w == 1) {
-        float sa = 0.0f;
-#pragma unroll
-        for (int c = 0; c < CPL; ++c) sa += fabsf(xv.v[c]);
-        sa = warp_sum(sa);
-        out.scale = f16_bits(__fdiv_rn(sa, static_cast<float>(DV)));
-#pragma unroll
-        for (int c = 0; c < CPL; ++c) u[c] = xv.v[c] < 0.0f ? 1u : 0u;
-    } else if (w >= 2) {
-        const int n = (1 << (w - 1)) - 1;
-        const float nf = static_cast<float>(n);
-        const float inv_n = __frcp_rn(nf);
-        const float R = out.R;
-        if (R == 0.0f) {
-            if (refit) out.fidx = kNFit - 1;
-#pragma unroll
-            for (int c = 0; c < CPL; ++c) u[c] = static_cast<uint32_t>(n);
-        } else {
-            if (refit) {
-                // lane l prepares candidate l & 15; every lane scores all 16 on its elements
-                const float Dl = cand_step(fit_factor(lane & 15), R, inv_n);
-                const float il = step_rcp(Dl);
-                float sse[16];
-#pragma unroll
-                for (int k = 0; k < 16; ++k) {
-                    const float D = __shfl_sync(kFull, Dl, k);
-                    const float inv = __shfl_sync(kFull, il, k);
-                    float acc = 0.0f;
-#pragma unroll
-                    for (int c = 0; c < CPL; ++c) {
-                        const float a = fabsf(xv.v[c]);
-                        const float tq = fminf(__fadd_rn(__fmul_rn(a, inv), kMagic), kMagic + nf);
-                        const float e = fmaf(-__fsub_rn(tq, kMagic), D, a);
-                        acc = fmaf(e, e, acc);
-                    }
-                    sse[k] = acc;
-                }
-                const float tot = reduce16(sse, lane);
-                const unsigned sb = __float_as_uint(tot);
-                const unsigned mn = __reduce_min_sync(kFull, sb);
-                const unsigned best = __reduce_max_sync(kFull, sb == mn ? ((lane >> 1) & 15) + 1 : 0u);
-                out.fidx = static_cast<int>(best) - 1;
-            }
-            const float D = cand_step(fit_factor(out.fidx), R, inv_n);
-            const float inv = step_rcp(D);
-            out.scale = f16_bits(D);
-#pragma unroll
-            for (int c = 0; c < CPL; ++c) {
-                const float tq = code_magic(xv.v[c], inv, kMagic - nf, kMagic + nf);
-                u[c] = __float_as_uint(tq) - (kMagicBits - static_cast<uint32_t>(n));
-            }
-        }
-    } else {
-#pragma unroll
-        for (int c = 0; c < CPL; ++c) u[c] = 0u;
-    }
-    store_codes<CPL>(row, lane, w, u);
-    return out;
+    for (int c = 0; c < CPL; ++c) chunk |= static_cast<uint64_t>(u[c]) << (c * w);
+    const int P = lane * CPL * w;
+    const int idx = P >> 5, sh = P & 31;
+    const uint64_t lo = chunk << sh;
+    const uint32_t hi = sh ? static_cast<uint32_t>(chunk >> (64 - sh)) : 0u;
+    const uint32_t w0 = static_cast<uint32_t>(lo), w1 = static_cast<uint32_t>(lo >> 32);
+    if (w0) atomicOr(words + idx, w0);
+    if (w1) atomicOr(words + idx + 1, w1);
+    if (hi) atomicOr(words + idx + 2, hi);
 }
 
 template <int DK, int DV, bool HEAD, bool SRC_PACKED, bool DST_PACKED>
@@ -162,6 +106,11 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
 
     // ---- 1. metadata ---------------------------------------------------------------------
     if (tid == 0) sm.flag = 0;
+    if (tid < kNFit) sm.fitf[tid] = fit_factor(tid);
+    if (tid >= 32 && tid < 32 + 17) {
+        const int w = tid - 32;
+        sm.inv_n[w] = w >= 2 ? __frcp_rn(static_cast<float>((1 << (w - 1)) - 1)) : 0.0f;
+    }
     if (SRC_PACKED) {
         for (int i = tid; i < DK; i += 256) sm.w_in[i] = HEAD ? p.in_widths[bh] : p.in_widths[ubase + i];
         for (int g = tid; g < NSG; g += 256) sm.scale_in[g] = f16_value(p.in_scales[gbase + g]);
@@ -215,6 +164,16 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
                 atomicExch(&sm.flag, 1);
         }
     }
+    if (SRC_PACKED && !HEAD && tid >= 64 && tid < 64 + DK) {
+        // per-row dequantisation x = (float(u) - A) S + Bc: w >= 2 -> (q) Delta; w = 1 -> +-m;
+        // w = 0 -> 0 (float(u) is 2^23 + u built from the code bits)
+        const int i = tid - 64;
+        const int w = min(static_cast<int>(sm.w_in[i]), 16);
+        const float D = sm.scale_in[i];
+        sm.deqA[i] = 8388608.0f + static_cast<float>(w >= 2 ? (1 << (w - 1)) - 1 : 0);
+        sm.deqS[i] = w >= 2 ? D : (w == 1 ? -2.0f * D : 0.0f);
+        sm.deqB[i] = w == 1 ? D : 0.0f;
+    }
     __syncthreads();
     if (sm.flag) {
         if (tid == 0) raise_status(p.status, QS_DEV_LAYOUT);
@@ -243,11 +202,16 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
             const int w = sm.w_in[i];
             uint32_t u[CPL];
             extract_codes<CPL>(pay + sm.off_in[i], lane, w, u);
-            const float nf2 = 8388608.0f + static_cast<float>(w >= 2 ? (1 << (w - 1)) - 1 : 0);
+            if (!HEAD) {
+                const float A = sm.deqA[i], S = sm.deqS[i], Bc = sm.deqB[i];
 #pragma unroll
-            for (int c = 0; c < CPL; ++c) {
-                const float D = HEAD ? sm.scale_in[(i >> 5) * DV + lane * CPL + c] : sm.scale_in[i];
-                x[r][c] = dequant(u[c], w, D, nf2);
+                for (int c = 0; c < CPL; ++c)
+                    x[r][c] = fmaf(__fsub_rn(__uint_as_float(kTwo23Bits | u[c]), A), S, Bc);
+            } else {
+                const float nf2 = 8388608.0f + static_cast<float>(w >= 2 ? (1 << (w - 1)) - 1 : 0);
+#pragma unroll
+                for (int c = 0; c < CPL; ++c)
+                    x[r][c] = dequant(u[c], w, sm.scale_in[(i >> 5) * DV + lane * CPL + c], nf2);
             }
         } else if (p.dense_in != nullptr) {
             const float* src = p.dense_in + (static_cast<size_t>(bh) * DK + i) * DV + lane * CPL;
@@ -264,9 +228,15 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
         }
     }
     if (SRC_PACKED) __syncthreads();   // the staging buffer is reused for the output rows
+    if (DST_PACKED) {                  // zero the output rows: codes are OR-ed in
+        const int nz = (sm.off_out[DK] + 16) / 16;
+        for (int i = tid; i < nz; i += 256) reinterpret_cast<uint4*>(pay)[i] = make_uint4(0, 0, 0, 0);
+        if (!has_tokens) __syncthreads();
+    }
 
     // ---- 4. tokens of this write-back interval (Eq. 1) --------------------------------------
     for (int t = p.t_begin; t < p.t_end; ++t) {
+        if (t > p.t_begin) __syncthreads();   // every warp is done with the previous token's k, u
         const size_t tok = (static_cast<size_t>(b) * p.T + t) * p.H + h;
         const float beta = p.erase ? __ldg(p.beta + tok) : 1.0f;
         float rate_h = 0.0f;
@@ -375,19 +345,106 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
     if (DST_PACKED) {
         const bool refit = (p.fit_every <= 1) || ((p.w_index + h) % p.fit_every == 0);
         if (!HEAD) {
+            // (a) row ranges (and 1-bit means) by warp reductions
 #pragma unroll
             for (int r = 0; r < RPW; ++r) {
                 const int i = warp * RPW + r;
-                RowVals<CPL> xv;
+                float amax = 0.0f, asum = 0.0f;
 #pragma unroll
-                for (int c = 0; c < CPL; ++c) xv.v[c] = x[r][c];
-                const RowOut o = quantise_row<CPL, DV>(xv, sm.w_out[i], lane, refit, sm.fidx_in[i],
-                                                       pay + sm.off_out[i]);
-                if (lane == 0) {
-                    if (p.range != nullptr) p.range[ubase + i] = o.R;
-                    p.out_scales[gbase + i] = static_cast<uint16_t>(o.scale);
-                    p.out_fidx[gbase + i] = static_cast<uint8_t>(o.fidx);
+                for (int c = 0; c < CPL; ++c) {
+                    amax = fmaxf(amax, fabsf(x[r][c]));
+                    asum += fabsf(x[r][c]);
                 }
+                const float R = warp_absmax(amax);
+                if (sm.w_out[i] == 1) asum = warp_sum(asum);
+                if (lane == 0) {
+                    sm.rowR[i] = R;
+                    sm.rowM[i] = asum;
+                }
+            }
+            __syncthreads();
+            // (b) scalar per-row work, one thread per row
+            if (tid < DK) {
+                const int i = tid, w = sm.w_out[i];
+                const float R = sm.rowR[i];
+                float D = 0.0f, inv = 0.0f;
+                int fidx = sm.fidx_in[i], mode = 0;
+                if (w == 1) {
+                    D = f16_round(__fdiv_rn(sm.rowM[i], static_cast<float>(DV)));
+                } else if (w >= 2) {
+                    const float inv_n = sm.inv_n[w];
+                    if (R == 0.0f) {
+                        if (refit) fidx = kNFit - 1;
+                    } else if (refit) {
+                        mode = 1;
+#pragma unroll 4
+                        for (int k = 0; k < kNFit; ++k) {
+                            const float Dk = cand_step(sm.fitf[k], R, inv_n);
+                            sm.cand[i][k][0] = Dk;
+                            sm.cand[i][k][1] = step_rcp(Dk);
+                        }
+                    } else {
+                        D = cand_step(sm.fitf[fidx], R, inv_n);
+                        inv = step_rcp(D);
+                    }
+                }
+                sm.rowD[i] = D;
+                sm.rowInv[i] = inv;
+                sm.mode[i] = static_cast<uint8_t>(mode);
+                sm.out_fidx[i] = static_cast<uint8_t>(fidx);
+            }
+            __syncthreads();
+            // (c) per row: factor search, codes, bits into the staging row
+#pragma unroll
+            for (int r = 0; r < RPW; ++r) {
+                const int i = warp * RPW + r;
+                const int w = sm.w_out[i];
+                uint32_t u[CPL];
+                if (w >= 2) {
+                    const int n = (1 << (w - 1)) - 1;
+                    const float nf = static_cast<float>(n);
+                    float D = sm.rowD[i], inv = sm.rowInv[i];
+                    if (sm.mode[i]) {
+                        const float4* ct = reinterpret_cast<const float4*>(&sm.cand[i][0][0]);
+                        float sse[16];
+#pragma unroll
+                        for (int kk = 0; kk < 8; ++kk) {
+                            const float4 cd = ct[kk];
+                            float a0 = 0.0f, a1 = 0.0f;
+#pragma unroll
+                            for (int c = 0; c < CPL; ++c) {
+                                const float a = fabsf(x[r][c]);
+                                const float t0 = fminf(__fadd_rn(__fmul_rn(a, cd.y), kMagic), kMagic + nf);
+                                const float e0 = fmaf(-__fsub_rn(t0, kMagic), cd.x, a);
+                                a0 = fmaf(e0, e0, a0);
+                                const float t1 = fminf(__fadd_rn(__fmul_rn(a, cd.w), kMagic), kMagic + nf);
+                                const float e1 = fmaf(-__fsub_rn(t1, kMagic), cd.z, a);
+                                a1 = fmaf(e1, e1, a1);
+                            }
+                            sse[2 * kk] = a0;
+                            sse[2 * kk + 1] = a1;
+                        }
+                        const float tot = reduce16(sse, lane);
+                        const unsigned sb = __float_as_uint(tot);
+                        const unsigned mn = __reduce_min_sync(kFull, sb);
+                        const int best = static_cast<int>(
+                                             __reduce_max_sync(kFull, sb == mn ? ((lane >> 1) & 15) + 1 : 0u)) - 1;
+                        D = sm.cand[i][best][0];
+                        inv = sm.cand[i][best][1];
+                        if (lane == 0) sm.out_fidx[i] = static_cast<uint8_t>(best);
+                    }
+                    if (lane == 0) sm.out_scale[i] = f16_bits(D);
+#pragma unroll
+                    for (int c = 0; c < CPL; ++c) {
+                        const float tq = code_magic(x[r][c], inv, kMagic - nf, kMagic + nf);
+                        u[c] = __float_as_uint(tq) - (kMagicBits - static_cast<uint32_t>(n));
+                    }
+                } else {
+                    if (lane == 0) sm.out_scale[i] = f16_bits(sm.rowD[i]);
+#pragma unroll
+                    for (int c = 0; c < CPL; ++c) u[c] = (w == 1 && x[r][c] < 0.0f) ? 1u : 0u;
+                }
+                or_codes<CPL>(reinterpret_cast<uint32_t*>(pay + sm.off_out[i]), lane, w, u);
             }
         } else {
             // head unit: one width per head; scale groups = 32 key rows x one value column.
@@ -418,7 +475,7 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
             if (w >= 2) {
                 n = (1u << (w - 1)) - 1u;
                 nf = static_cast<float>(n);
-                inv_n = __frcp_rn(nf);
+                inv_n = sm.inv_n[w];
             }
             if (w >= 2 && refit) {
                 float best[CPL];
@@ -430,7 +487,7 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
                 for (int round = 0; round < 4; ++round) {
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk) {
-                        const float f = fit_factor(round * 4 + kk);
+                        const float f = sm.fitf[round * 4 + kk];
 #pragma unroll
                         for (int c = 0; c < CPL; ++c) {
                             const float D = cand_step(f, R[c], inv_n);
@@ -467,7 +524,7 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
 #pragma unroll
             for (int c = 0; c < CPL; ++c) {
                 if (w >= 2) {
-                    Dc[c] = (R[c] == 0.0f) ? 0.0f : cand_step(fit_factor(fc[c]), R[c], inv_n);
+                    Dc[c] = (R[c] == 0.0f) ? 0.0f : cand_step(sm.fitf[fc[c]], R[c], inv_n);
                 } else if (w == 1) {
                     Dc[c] = f16_round(__fdiv_rn(R[c], 32.0f));
                 } else {
@@ -490,14 +547,14 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
                         u[c] = 0u;
                     }
                 }
-                store_codes<CPL>(pay + sm.off_out[i], lane, w, u);
+                or_codes<CPL>(reinterpret_cast<uint32_t*>(pay + sm.off_out[i]), lane, w, u);
             }
             if ((warp & 1) == 0) {
 #pragma unroll
                 for (int c = 0; c < CPL; ++c) {
                     const int g = blk * DV + lane * CPL + c;
-                    p.out_scales[gbase + g] = f16_bits(Dc[c]);
-                    p.out_fidx[gbase + g] = static_cast<uint8_t>(fc[c]);
+                    sm.out_scale[g] = f16_bits(Dc[c]);
+                    sm.out_fidx[g] = static_cast<uint8_t>(fc[c]);
                 }
             }
         }
@@ -508,6 +565,12 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
         const Vec* srcv = reinterpret_cast<const Vec*>(pay);
         const int nv = nbytes / static_cast<int>(sizeof(Vec));
         for (int i = tid; i < nv; i += 256) dst[i] = srcv[i];
+        for (int g = tid; g < NSG; g += 256) {
+            p.out_scales[gbase + g] = sm.out_scale[g];
+            p.out_fidx[gbase + g] = sm.out_fidx[g];
+        }
+        if (!HEAD && p.range != nullptr)
+            for (int i = tid; i < DK; i += 256) p.range[ubase + i] = sm.rowR[i];
     } else if (p.dense_out != nullptr) {
 #pragma unroll
         for (int r = 0; r < RPW; ++r) {
@@ -551,7 +614,8 @@ cudaError_t launch_step_t(const qstate_cfg& cfg, const StepParams& p, cudaStream
 template <int DK, int DV>
 cudaError_t launch_step_shape(const qstate_cfg& cfg, int src_packed, int dst_packed,
                               const StepParams& p, cudaStream_t stream) {
-    const bool head = cfg.unit_kind == QSTATE_UNIT_HEAD;
+    // the allocation unit only shapes packing: dense -> dense runs the row-unit instance
+    const bool head = cfg.unit_kind == QSTATE_UNIT_HEAD && (src_packed || dst_packed);
 #define QS_CASE(HD, SP, DP)                                                            \
     if (head == HD && (src_packed != 0) == SP && (dst_packed != 0) == DP)              \
         return launch_step_t<DK, DV, HD, SP, DP>(cfg, p, stream);
