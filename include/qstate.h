@@ -162,6 +162,22 @@ int qstate_unpack(const qstate_cfg* cfg, const qstate_buf* in, float* S_out, voi
 int qstate_quant_decay(const qstate_cfg* cfg, const float* s, int32_t T, uint8_t* code_out,
                        float* lut_out, float* thr_out, void* stream);
 
+/* Same computation and outputs as qstate_quant_decay, for callers that cannot allocate device
+ * memory: code running where a device allocation is not allowed or would stall (inside a host
+ * framework whose allocator owns all device memory, a plugin that only receives its inputs and
+ * outputs, a latency-critical loop that must not call into the allocator).  The paper has no
+ * counterpart; it is a deployment convenience.  The thresholds, which qstate_quant_decay writes
+ * to thr_out, are kept instead in one fixed array inside the library: at most 65536 thresholds,
+ * i.e. channels x (2^gate_bits - 1) <= 65536 (4096 channels at gate_bits = 4); larger
+ * configurations return QSTATE_EINVAL with a message and launch nothing.  This call allocates
+ * nothing.  The array exists once per device for the life of the process; the first call with a
+ * device current looks its address up on the host, so make that first call before any stream
+ * capture.  Every call on a device shares the array and leaves its thresholds there; each call
+ * rewrites all the entries it reads before reading them, so nothing needs clearing, but calls
+ * whose kernels overlap on the GPU (for instance on two streams) race on it. */
+int qstate_quant_decay_noalloc(const qstate_cfg* cfg, const float* s, int32_t T,
+                               uint8_t* code_out, float* lut_out, void* stream);
+
 /* One write-back interval: tokens [t_begin, t_end) (at most C of them) of every head, from the
  * state packed in `in` to `out` (whose widths and offsets must already hold the target
  * allocation).  Unpack + dequantise, decay, delta update and readout o_t (device,

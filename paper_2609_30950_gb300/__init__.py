@@ -52,7 +52,8 @@ class _Inputs(ct.Structure):
 
 EXPORTS = ["qstate_validate", "qstate_region_bytes", "qstate_units", "qstate_scale_groups",
            "qstate_bits_per_element", "qstate_init", "qstate_alloc_bits", "qstate_pack",
-           "qstate_unpack", "qstate_quant_decay", "qstate_step", "qstate_scan",
+           "qstate_unpack", "qstate_quant_decay", "qstate_quant_decay_noalloc", "qstate_step",
+           "qstate_scan",
            "qstate_scan_fp32", "qstate_check", "qstate_last_error"]
 
 _lib = None
@@ -88,6 +89,7 @@ def load(path: str | None = None, build_if_missing: bool = False):
     L.qstate_pack.argtypes = [PC, P, ct.POINTER(_Buf), P, P]
     L.qstate_unpack.argtypes = [PC, ct.POINTER(_Buf), P, P]
     L.qstate_quant_decay.argtypes = [PC, P, ct.c_int32, P, P, P, P]
+    L.qstate_quant_decay_noalloc.argtypes = [PC, P, ct.c_int32, P, P, P]
     L.qstate_step.argtypes = [PC, ct.POINTER(_Buf), ct.POINTER(_Buf), ct.POINTER(_Inputs),
                               ct.c_int32, ct.c_int32, ct.c_int32, P, ct.POINTER(_Stats), P]
     L.qstate_scan.argtypes = [PC, ct.POINTER(_Buf), ct.POINTER(_Buf), ct.POINTER(_Inputs),
@@ -273,6 +275,14 @@ def qstate_quant_decay(cfg: Config, s, code_out, lut_out, thr_out, stream=None) 
     c = cfg.c()
     _check(_lib_or_raise().qstate_quant_decay(ct.byref(c), _ptr(s), int(s.shape[1]), _ptr(code_out),
                                               _ptr(lut_out), _ptr(thr_out), _stream(stream)))
+
+
+def qstate_quant_decay_noalloc(cfg: Config, s, code_out, lut_out, stream=None) -> None:
+    """qstate_quant_decay without a threshold buffer (see include/qstate.h)."""
+    c = cfg.c()
+    _check(_lib_or_raise().qstate_quant_decay_noalloc(ct.byref(c), _ptr(s), int(s.shape[1]),
+                                                      _ptr(code_out), _ptr(lut_out),
+                                                      _stream(stream)))
 
 
 def qstate_step(cfg: Config, src: State, dst: State, x: Inputs, t_begin: int, t_end: int,

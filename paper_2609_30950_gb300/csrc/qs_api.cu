@@ -330,6 +330,31 @@ int qstate_quant_decay(const qstate_cfg* cfg, const float* s, int32_t T, uint8_t
     return e == cudaSuccess ? QSTATE_OK : cuda_fail(e, "decay quantiser");
 }
 
+int qstate_quant_decay_noalloc(const qstate_cfg* cfg, const float* s, int32_t T, uint8_t* code_out,
+                               float* lut_out, void* stream) {
+    int rc = validate(cfg);
+    if (rc) return rc;
+    if (cfg->gate_bits < 1) return fail(QSTATE_EINVAL, "gate_bits must be >= 1");
+    if (!s || !code_out || !lut_out || T < 1) return fail(QSTATE_EINVAL, "null pointer or T < 1");
+    const int nchan = cfg->decay_kind == QSTATE_DECAY_ROW ? cfg->H * cfg->dk : cfg->H;
+    const long long need = static_cast<long long>(nchan) * ((1 << cfg->gate_bits) - 1);
+    if (need > quant_decay_scratch_capacity())
+        return fail(QSTATE_EINVAL,
+                    "qstate_quant_decay_noalloc: %lld thresholds (%d channels x %d) exceed the "
+                    "built-in scratch of %lld; use qstate_quant_decay with a caller buffer",
+                    need, nchan, (1 << cfg->gate_bits) - 1, quant_decay_scratch_capacity());
+    cudaError_t e;
+    int* status = status_word(&e);
+    if (!status) return cuda_fail(e, "status word");
+    float* thr = nullptr;
+    e = quant_decay_scratch(&thr);
+    if (e != cudaSuccess) return cuda_fail(e, "threshold scratch lookup");
+    const long long count = static_cast<long long>(cfg->B) * T;
+    e = launch_quant_decay(s, count, nchan, cfg->gate_bits, code_out, lut_out, thr, status,
+                           static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? QSTATE_OK : cuda_fail(e, "decay quantiser");
+}
+
 int qstate_step(const qstate_cfg* cfg, qstate_buf* in, qstate_buf* out, const qstate_inputs* x,
                 int32_t t_begin, int32_t t_end, int32_t w_index, float* o, qstate_stats* stats,
                 void* stream) {

@@ -8,6 +8,7 @@
 //      (l_0 = min and l_{L-1} = max exactly);
 //   3. codes = number of thresholds <= s, one byte per rate, 16 rates per thread-iteration.
 #include <algorithm>
+#include <mutex>
 
 #include "qs_common.cuh"
 
@@ -131,6 +132,39 @@ cudaError_t launch_quant_decay(const float* s, long long count, int nchan, int g
         decay_codes_generic_kernel<<<blocks, 256, 0, stream>>>(s, total, nchan, L - 1, thr, codes);
     }
     return cudaGetLastError();
+}
+
+// ---- variant without caller-supplied threshold buffer -------------------------------------------
+// The thresholds are an intermediate of the quantiser.  Callers that must not allocate device
+// memory of their own keep them here: one file-scope array per device (every GPU that loads
+// the library holds it until the process exits), shared by all calls on that device.
+constexpr long long kDecayScratchFloats = 65536;   // 256 KiB: channels x (2^g - 1) thresholds
+static __device__ __align__(256) float g_decay_thr_scratch[kDecayScratchFloats];
+
+namespace {
+constexpr int kMaxDev = 64;
+std::mutex g_scratch_mu;
+float* g_scratch_addr[kMaxDev] = {};
+}  // namespace
+
+long long quant_decay_scratch_capacity() { return kDecayScratchFloats; }
+
+// Device address of the threshold scratch on the current device, looked up on the first call
+// made with that device current (a host-side lookup: make it before any stream capture).
+cudaError_t quant_decay_scratch(float** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDev) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(g_scratch_mu);
+    if (!g_scratch_addr[dev]) {
+        void* ptr = nullptr;
+        e = cudaGetSymbolAddress(&ptr, g_decay_thr_scratch);
+        if (e != cudaSuccess) return e;
+        g_scratch_addr[dev] = static_cast<float*>(ptr);
+    }
+    *out = g_scratch_addr[dev];
+    return cudaSuccess;
 }
 
 }  // namespace qs

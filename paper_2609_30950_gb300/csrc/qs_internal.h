@@ -79,5 +79,7 @@ cudaError_t launch_alloc(const AllocParams& p, cudaStream_t stream);
 cudaError_t launch_quant_decay(const float* s, long long count, int nchan, int g,
                                uint8_t* codes, float* lut, float* thr, int* status,
                                cudaStream_t stream);
+long long quant_decay_scratch_capacity();
+cudaError_t quant_decay_scratch(float** out);
 
 }  // namespace qs
