@@ -8,6 +8,6 @@ cudaError_t launch_step_128x128(const qstate_cfg& cfg, int src_packed, int dst_p
     return launch_step_shape<128, 128>(cfg, src_packed, dst_packed, p, stream);
 }
 cudaError_t launch_wb_row_128x128(const qstate_cfg& cfg, const StepParams& p, cudaStream_t stream) {
-    return launch_wb_row_t<128, 128, 16>(cfg, p, stream);
+    return launch_wb_row_t<128, 128, 8>(cfg, p, stream);
 }
 }  // namespace qs

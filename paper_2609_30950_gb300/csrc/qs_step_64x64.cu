@@ -8,6 +8,6 @@ cudaError_t launch_step_64x64(const qstate_cfg& cfg, int src_packed, int dst_pac
     return launch_step_shape<64, 64>(cfg, src_packed, dst_packed, p, stream);
 }
 cudaError_t launch_wb_row_64x64(const qstate_cfg& cfg, const StepParams& p, cudaStream_t stream) {
-    return launch_wb_row_t<64, 64, 16>(cfg, p, stream);
+    return launch_wb_row_t<64, 64, 8>(cfg, p, stream);
 }
 }  // namespace qs

@@ -3,25 +3,32 @@
 // The hot path of qstate_step / qstate_scan for per-row widths (KDA, Mamba-2): one write-back
 // interval of every head, packed state in, packed state out.
 //
-// Each CTA (NW warps, one CTA per SM) walks heads g = blockIdx.x, blockIdx.x + gridDim.x, ...
-// While it works on head g, cp.async copies head g + gridDim.x's inputs into the other half of
-// a double buffer: widths in/out, FP16 scales, fitted-factor indices, EMA statistics, the first
-// token's k, q, v and rates, and the head's packed rows (whose byte window comes from offsets
-// fetched one head earlier).  Warp w owns key rows [w RPW, (w+1) RPW), lane l the value
-// columns [l CPL, (l+1) CPL).  Per head there are five CTA barriers:
+// Each CTA (NW = 8 warps, two CTAs per SM so that one's barriers and latencies overlap the
+// other's work) walks a contiguous block of heads.  While it works on head g, cp.async copies
+// head g + 1's metadata into the other half of a double buffer (widths in/out, FP16 scales,
+// fitted-factor indices, EMA statistics, the first token's k, q, v, rates and their level table)
+// and, once head g is unpacked, head g + 1's packed rows into the single payload buffer (their
+// byte window comes from offsets fetched one head earlier).
+//
+// Two thread layouts share the head's FP32 state through a shared-memory buffer (16-byte
+// groups XOR-swizzled per row):
+//  * row layout: TPR = dv/32 lanes per row, each owning 32 consecutive value columns, i.e. a
+//    word-aligned run of 32 codes (4w bytes).  Warps take rows in order of width (a counting
+//    sort per head), so the code arithmetic of a warp is specialised for one width.  Used to
+//    unpack + dequantise and for the write-back (range, factor search, codes, packing).
+//  * update layout: warp w owns key rows [w RPW, (w+1) RPW), lane l the value columns
+//    [l CPL, (l+1) CPL), so the reductions of Eq. (1) over key rows stay in registers.
+// Per head there are seven CTA barriers:
 //   B1  the head's inputs have landed            -> issue the next head's copies
-//   B2  prep: row offsets (prefix sums of widths), layout checks, per-row decay, EMA update,
-//       dequantisation constants with the first token's decay folded in, erase vector, k.q
-//       -> unpack + dequantise into registers (column pairs), Eq. (1) partial p = a^T S',
-//       r = q^T S' per lane over the warp's rows
-//   B3  partials of all warps                     -> u = beta v - p, o = r + u (k.q)
-//   B4  u                                         -> S = S' + k u^T; then, warp-locally:
-//       row ranges, per-row steps (lane r <-> row r) or the 16 candidate steps of every row
-//       (4 (row, candidate) pairs per lane), the squared-error search (candidates outer,
-//       rows inner, packed FP32), codes folded into 64-bit chunks, and each group of lanes
-//       holding 8 consecutive codes writing their w bytes into the output staging rows
-//   B5  all rows staged                           -> vector store of the head's region and
-//       coalesced stores of scales, factor indices, ranges and EMAs.
+//   B2  prep: row offsets (prefix sums of widths), rows sorted by width, layout checks,
+//       per-row decay, EMA update, dequantisation constants with the first token's decay
+//       folded in, erase vector, k.q                -> unpack (row layout) into the buffer
+//   B3  -> registers (update layout); partials p = a^T S', r = q^T S'
+//   B4  -> u = beta v - p, o = r + u (k.q)
+//   B5  -> S = S' + k u^T (further tokens of the interval repeat B3..B5), state to the buffer
+//   B6  -> write-back (row layout): row range R, the 16 candidate steps and their squared
+//       errors (refit), codes, and each lane's packed words stored to the output region
+//   B7  -> coalesced stores of scales, factor indices, ranges and EMAs.
 // The next head's B1 orders the reuse of stage and staging buffers.
 #pragma once
 
@@ -42,54 +49,54 @@ struct alignas(16) WbStage {
     uint16_t sc_in[DK];
     float ms[DK], mr[DK], k[DK], q[DK], s[DK];
     float v[DV];
+    float lut[DK * 4];                           // the head's decay levels (when 2^g <= 4)
     float beta, rate_h, pad0, pad1;
     int in_off, in_end, out_off, ok;              // payload window of this head
     int nxt_in_off, nxt_in_end, nxt_out_off, pad2;   // offsets of the following head
 };
 
 template <int DK, int DV, int NW>
+struct WbGeom {
+    static constexpr int RPW = DK / NW;       // update layout: rows per warp
+    static constexpr int CPL = DV / 32;       // update layout: columns per lane
+    static constexpr int TPR = DV / 32;       // row layout: lanes per row
+    static constexpr int RPB = 32 / TPR;      // row layout: rows per warp
+    static constexpr int KPT = kNFit / TPR;   // candidate steps each lane of a row prepares
+};
+
+template <int DK, int DV, int NW>
 struct alignas(16) WbSmem {
-    static constexpr int RPW = DK / NW;
     WbStage<DK, DV> st[2];
-    float cand[DK][kNFit][2];             // (Delta_k, 1/Delta_k) per row and candidate
-    uint2 chunk[NW][RPW][32];             // each lane's codes per row
-    float red[2][NW][DV];                 // p and r partials per warp
+    float sbuf[DK * DV];                  // FP32 state of the head (swizzled rows)
+    union {
+        float red[2][NW][DV];             // p and r partials per warp (token phase)
+        float2 cand[NW][32 / (DV / 32)][kNFit];   // per warp and row: (1/Delta_k, -Delta_k)
+    } rc;
     float4 deq[DK];                       // (-A, S, B, 0): x = (2^23 + u - A) S + B
     float4 wc[17];                        // per width: (n, 1/n, 2^23*1.5 - n, 2^23*1.5 + n)
     float tk[DK], tq[DK], tv[DV];         // inputs of tokens after the first (C > 1)
     float a[DK], d[DK];                   // erase vector beta k, decay of the current token
     float u[DV];
-    float rowR[DK], rowM[DK];
+    float rowR[DK];
     float fitf[kNFit];
     float wsum[NW];
-    int best_k[DK];
     int off_in[DK + 1], off_out[DK + 1];
+    int cnt[2][17];
+    uint8_t ord_in[DK], ord_out[DK];      // rows in order of input / output width
     uint16_t out_scale[DK];
     uint8_t out_fidx[DK];
     int flag;
 };
 
-// Sum N per-lane values over the warp by recursive halving; lane l ends with the total of
-// value index (l >> (5 - log2 N)) & (N - 1).
-template <int N>
-__device__ __forceinline__ float reduce_rows(float (&v)[N], int lane) {
-    constexpr int LOG = N == 16 ? 4 : N == 8 ? 3 : N == 4 ? 2 : N == 2 ? 1 : 0;
-#pragma unroll
-    for (int st = 0; st < LOG; ++st) {
-        const int half = (N / 2) >> st;
-        const int off = 16 >> st;
-        const bool upper = (lane & off) != 0;
-#pragma unroll
-        for (int i = 0; i < half; ++i) {
-            const float send = upper ? v[i] : v[i + half];
-            const float keep = upper ? v[i + half] : v[i];
-            v[i] = keep + __shfl_xor_sync(kFull, send, off);
-        }
-    }
-    float t = v[0];
-#pragma unroll
-    for (int off = 16 >> LOG; off > 0; off >>= 1) t += __shfl_xor_sync(kFull, t, off);
-    return t;
+// Float offset of 16-byte group G of row i in the state buffer.  The XOR keeps each group in
+// its block of 8 and spreads, over the 32 banks, the groups that one 8-lane phase touches in
+// the update layout (one row) and, for two rows of different parity, in the row layout.
+template <int DV>
+__device__ __forceinline__ int sb_off(int i, int G) {
+    int s;
+    if constexpr (DV == 128) s = ((G >> 3) & 3) | ((i & 1) << 2);
+    else s = ((G >> 3) & 1) | ((i & 3) << 1);
+    return i * DV + 4 * (G ^ s);
 }
 
 __device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
@@ -107,68 +114,142 @@ __device__ __forceinline__ void cp_async4(void* smem, const void* gmem) {
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
 
-// ---- packing of one row: 8 consecutive codes (w bits each) = w bytes -------------------------
-// Lanes own CPL consecutive codes; groups of 8 / CPL lanes gather their chunks by shuffles and
-// the group's first lane stores the w bytes at byte w * group with aligned stores.
-// ALIGN16: dst is 16-byte aligned when NB == 16 (rows of dv = 128 start on 16 bytes).
-template <int NB, bool ALIGN16>
-__device__ __forceinline__ void store_bytes(uint8_t* dst, uint64_t lo, uint64_t hi) {
-    if constexpr (NB == 16 && ALIGN16) {
-        *reinterpret_cast<uint4*>(dst) = make_uint4(static_cast<uint32_t>(lo), static_cast<uint32_t>(lo >> 32),
-                                                   static_cast<uint32_t>(hi), static_cast<uint32_t>(hi >> 32));
-    } else if constexpr (NB == 8) {
-        *reinterpret_cast<uint2*>(dst) = make_uint2(static_cast<uint32_t>(lo), static_cast<uint32_t>(lo >> 32));
-    } else if constexpr (NB % 4 == 0) {
-#pragma unroll
-        for (int k = 0; k < NB / 4; ++k) {
-            const uint64_t s = k < 2 ? lo : hi;
-            reinterpret_cast<uint32_t*>(dst)[k] = static_cast<uint32_t>(s >> ((k & 1) * 32));
-        }
-    } else if constexpr (NB % 2 == 0) {
-#pragma unroll
-        for (int k = 0; k < NB / 2; ++k) {
-            const uint64_t s = k < 4 ? lo : hi;
-            reinterpret_cast<uint16_t*>(dst)[k] = static_cast<uint16_t>(s >> ((k & 3) * 16));
-        }
-    } else {
-#pragma unroll
-        for (int k = 0; k < NB; ++k) {
-            const uint64_t s = k < 8 ? lo : hi;
-            dst[k] = static_cast<uint8_t>(s >> ((k & 7) * 8));
-        }
-    }
+// ---- row layout: 32 consecutive codes of one row per lane ---------------------------------------
+// The lane's codes occupy the 4W bytes at byte 4 W q of the row (q = its part), a whole number of
+// words: code c of the run sits at bits [c W, c W + W) of those words.
+
+template <int W, int C>
+__device__ __forceinline__ uint32_t run_code(const uint32_t (&wd)[W + 1]) {
+    constexpr int bp = C * W, k = bp >> 5, sh = bp & 31;
+    constexpr uint32_t mask = (W >= 32) ? 0xffffffffu : ((1u << W) - 1u);
+    if constexpr (sh + W <= 32) return (wd[k] >> sh) & mask;
+    else return __funnelshift_r(wd[k], wd[k + 1], sh) & mask;
 }
 
-template <int CPL, int W>
-__device__ __forceinline__ void pack_row_w(uint8_t* row, int lane, uint64_t chunk) {
+template <int W, int C>
+struct RunDecode {
+    __device__ __forceinline__ static void go(const uint32_t (&wd)[W + 1], float2 (&v)[16], float2 A2, float2 S2, float2 B2) {
+        const float2 t = make_float2(__uint_as_float(kTwo23Bits | run_code<W, C>(wd)),
+                                     __uint_as_float(kTwo23Bits | run_code<W, C + 1>(wd)));
+        v[C / 2] = __ffma2_rn(__fadd2_rn(t, A2), S2, B2);
+        RunDecode<W, C + 2>::go(wd, v, A2, S2, B2);
+    }
+};
+template <int W>
+struct RunDecode<W, 32> {
+    __device__ __forceinline__ static void go(const uint32_t (&)[W + 1], float2 (&)[16], float2, float2, float2) {}
+};
+
+// Unpack + dequantise the lane's 32 codes (row i, part q) into the state buffer.
+template <int W, int DV>
+__device__ __forceinline__ void unpack_run(const uint8_t* src, const float4 dq, float* sb, int i, int q) {
+    float2 v[16];
+    const float2 A2 = make_float2(dq.x, dq.x), S2 = make_float2(dq.y, dq.y), B2 = make_float2(dq.z, dq.z);
     if constexpr (W == 0) {
-        return;
-    } else {
-        constexpr int G = 8 / CPL;          // lanes per 8 codes
-        constexpr int CB = CPL * W;         // bits per lane (<= 64)
-        uint64_t lo = chunk, hi = 0;
-        // gather: stage s merges pairs at distance 2^s, doubling the bit count
 #pragma unroll
-        for (int s = 0, d = 1; d < G; ++s, d <<= 1) {
-            const int sh = CB << s;         // bits held so far
-            const uint64_t olo = __shfl_down_sync(kFull, lo, d);
-            const uint64_t ohi = (2 * sh > 64) ? __shfl_down_sync(kFull, hi, d) : 0ull;
-            if (sh < 64) {
-                hi |= (olo >> (64 - sh)) | (ohi << sh);
-                lo |= olo << sh;
-            } else {
-                hi |= olo;
-            }
-        }
-        if ((lane % G) == 0) store_bytes<W, CPL == 4>(row + (lane / G) * W, lo, hi);
+        for (int k = 0; k < 16; ++k) v[k] = B2;
+    } else {
+        uint32_t wd[W + 1];
+#pragma unroll
+        for (int k = 0; k < W; ++k) wd[k] = reinterpret_cast<const uint32_t*>(src)[k];
+        wd[W] = 0u;
+        RunDecode<W, 0>::go(wd, v, A2, S2, B2);
+    }
+#pragma unroll
+    for (int g = 0; g < 8; ++g)
+        *reinterpret_cast<float4*>(sb + sb_off<DV>(i, 8 * q + g)) =
+            make_float4(v[2 * g].x, v[2 * g].y, v[2 * g + 1].x, v[2 * g + 1].y);
+}
+
+template <int DV>
+__device__ __forceinline__ void unpack_row(int w, const uint8_t* src, const float4 dq, float* sb, int i, int q) {
+    switch (w) {
+#define QS_W(N) case N: unpack_run<N, DV>(src, dq, sb, i, q); break;
+        QS_W(0) QS_W(1) QS_W(2) QS_W(3) QS_W(4) QS_W(5) QS_W(6) QS_W(7) QS_W(8)
+        QS_W(9) QS_W(10) QS_W(11) QS_W(12) QS_W(13) QS_W(14) QS_W(15) QS_W(16)
+#undef QS_W
+        default: break;
     }
 }
 
-// Store one row: `chunk` holds the lane's CPL codes, code c at bits [c w, c w + w).
-template <int CPL>
-__device__ __forceinline__ void pack_row(uint8_t* row, int lane, int w, uint64_t chunk) {
+// Packing.  With b_c the bit pattern of kMagic + q_c (= kMagicBits + q_c), the stored code is
+// u_c = q_c + n = b_c + (n - kMagicBits) (mod 2^32), so each word is a sum of b_c << sh_c plus a
+// per-word constant: one integer multiply-add per code (codes that straddle two words add their
+// high bits to the next word separately).
+template <int W>
+__host__ __device__ constexpr uint32_t run_pack_const(int k) {
+    uint32_t s = 0u;
+    const uint32_t C = static_cast<uint32_t>((1 << (W - 1)) - 1) - kMagicBits;
+    for (int c = 0; c < 32; ++c)
+        if (((c * W) >> 5) == k) s += C << ((c * W) & 31);
+    return s;
+}
+
+template <int W, int C>
+__device__ __forceinline__ void run_put(uint32_t (&wd)[W], uint32_t b) {
+    constexpr int bp = C * W, k = bp >> 5, sh = bp & 31;
+    constexpr uint32_t Cn = static_cast<uint32_t>((1 << (W - 1)) - 1) - kMagicBits;
+    wd[k] += b << sh;
+    if constexpr (sh + W > 32) wd[k + 1] += (b + Cn) >> (32 - sh);
+}
+
+template <int W, int C>
+struct RunEncode {
+    __device__ __forceinline__ static void go(uint32_t (&wd)[W], const float2 (&xv)[16], float2 i2, float lo, float hi) {
+        const float2 t = __fadd2_rn(__fmul2_rn(xv[C / 2], i2), make_float2(kMagic, kMagic));
+        run_put<W, C>(wd, __float_as_uint(fminf(fmaxf(t.x, lo), hi)));
+        run_put<W, C + 1>(wd, __float_as_uint(fminf(fmaxf(t.y, lo), hi)));
+        RunEncode<W, C + 2>::go(wd, xv, i2, lo, hi);
+    }
+};
+template <int W>
+struct RunEncode<W, 32> {
+    __device__ __forceinline__ static void go(uint32_t (&)[W], const float2 (&)[16], float2, float, float) {}
+};
+
+// MAXA: alignment of the row starts (16 bytes for dv = 128, 8 for dv = 64).
+template <int NWD, int MAXA>
+__device__ __forceinline__ void store_words(uint8_t* dst, const uint32_t (&wd)[NWD]) {
+    if constexpr (NWD % 4 == 0 && MAXA >= 16) {
+#pragma unroll
+        for (int k = 0; k < NWD; k += 4)
+            *reinterpret_cast<uint4*>(dst + 4 * k) = make_uint4(wd[k], wd[k + 1], wd[k + 2], wd[k + 3]);
+    } else if constexpr (NWD % 2 == 0) {
+#pragma unroll
+        for (int k = 0; k < NWD; k += 2) *reinterpret_cast<uint2*>(dst + 4 * k) = make_uint2(wd[k], wd[k + 1]);
+    } else {
+#pragma unroll
+        for (int k = 0; k < NWD; ++k) reinterpret_cast<uint32_t*>(dst)[k] = wd[k];
+    }
+}
+
+// Quantise + pack the lane's 32 values (row of width W) to dst (4W bytes at byte 4 W q of a row
+// aligned to MAXA bytes): q = clamp(rint(x / Delta), -n, n), offset binary.
+template <int W, int MAXA>
+__device__ __forceinline__ void pack_run(const float2 (&xv)[16], float inv, uint8_t* dst) {
+    if constexpr (W == 1) {
+        // sign bit, code 1 for x < 0 (negative zero counts as positive)
+        uint32_t wd[1] = {0u};
+#pragma unroll
+        for (int c = 0; c < 16; ++c) {
+            wd[0] |= (xv[c].x < 0.0f ? 1u : 0u) << (2 * c);
+            wd[0] |= (xv[c].y < 0.0f ? 2u : 0u) << (2 * c);
+        }
+        store_words<1, MAXA>(dst, wd);
+    } else if constexpr (W >= 2) {
+        constexpr float n = static_cast<float>((1 << (W - 1)) - 1);
+        uint32_t wd[W];
+#pragma unroll
+        for (int k = 0; k < W; ++k) wd[k] = run_pack_const<W>(k);
+        RunEncode<W, 0>::go(wd, xv, make_float2(inv, inv), kMagic - n, kMagic + n);
+        store_words<W, MAXA>(dst, wd);
+    }
+}
+
+template <int MAXA>
+__device__ __forceinline__ void pack_row(int w, const float2 (&xv)[16], float inv, uint8_t* dst) {
     switch (w) {
-#define QS_W(N) case N: pack_row_w<CPL, N>(row, lane, chunk); break;
+#define QS_W(N) case N: pack_run<N, MAXA>(xv, inv, dst); break;
         QS_W(1) QS_W(2) QS_W(3) QS_W(4) QS_W(5) QS_W(6) QS_W(7) QS_W(8)
         QS_W(9) QS_W(10) QS_W(11) QS_W(12) QS_W(13) QS_W(14) QS_W(15) QS_W(16)
 #undef QS_W
@@ -176,98 +257,113 @@ __device__ __forceinline__ void pack_row(uint8_t* row, int lane, int w, uint64_t
     }
 }
 
-// Issue the asynchronous copies of head g into stage S / payload buffer pay.  The head's
-// payload window (in_off, in_end) and output offset come from the previous stage (or, for the
-// first head, from direct loads); the window is checked before anything is copied.  One
+// Issue the asynchronous copies of head g's metadata into stage S.  The head's payload window
+// (in_off, in_end) and output offset come from the previous stage (or, for the first head, from
+// direct loads) and are checked here; gnext >= 0 names the head whose offsets to fetch.  One
 // commit group per call.
 template <int DK, int DV>
-__device__ __noinline__ void wb_issue(WbStage<DK, DV>& S, uint8_t* pay, int g, int in_off, int in_end,
-                                      int out_off, const WbParams& wp) {
+__device__ __noinline__ void wb_issue_meta(WbStage<DK, DV>& S, int g, int gnext, int in_off, int in_end,
+                                           int out_off, const WbParams& wp) {
     const StepParams& p = wp.s;
     const int tid = threadIdx.x;
     const bool stats = p.ema_s != nullptr;
     const int T = p.T;
-        const int b = g / p.H, h = g - (g / p.H) * p.H;
-        const size_t tok = (static_cast<size_t>(b) * T + p.t_begin) * p.H + h;
-        const size_t rb = static_cast<size_t>(g) * DK;
-        // fixed-size arrays, 16-byte chunks
-        constexpr int C8 = DK / 16, C16 = DK * 2 / 16, C32 = DK * 4 / 16, CV = DV * 4 / 16;
-        int c = tid;
-        if (c < C8) cp_async16(S.w_in + 16 * c, p.in_widths + rb + 16 * c);
-        else if ((c -= C8) < C8) cp_async16(S.w_out + 16 * c, p.out_widths + rb + 16 * c);
-        else if ((c -= C8) < C8) cp_async16(S.fidx + 16 * c, p.in_fidx + rb + 16 * c);
-        else if ((c -= C8) < C16) cp_async16(reinterpret_cast<uint8_t*>(S.sc_in) + 16 * c,
-                                             reinterpret_cast<const uint8_t*>(p.in_scales + rb) + 16 * c);
-        else if ((c -= C16) < C32) cp_async16(reinterpret_cast<uint8_t*>(S.k) + 16 * c,
-                                              reinterpret_cast<const uint8_t*>(p.k + tok * DK) + 16 * c);
-        else if ((c -= C32) < C32) cp_async16(reinterpret_cast<uint8_t*>(S.q) + 16 * c,
-                                              reinterpret_cast<const uint8_t*>(p.q + tok * DK) + 16 * c);
-        else if ((c -= C32) < CV) cp_async16(reinterpret_cast<uint8_t*>(S.v) + 16 * c,
-                                             reinterpret_cast<const uint8_t*>(p.v + tok * DV) + 16 * c);
-        else if ((c -= CV) < C32) {
-            if (stats) cp_async16(reinterpret_cast<uint8_t*>(S.ms) + 16 * c,
-                                  reinterpret_cast<const uint8_t*>(p.ema_s + rb) + 16 * c);
-        } else if ((c -= C32) < C32) {
-            if (stats) cp_async16(reinterpret_cast<uint8_t*>(S.mr) + 16 * c,
-                                  reinterpret_cast<const uint8_t*>(p.ema_r + rb) + 16 * c);
-        } else if ((c -= C32) < C32) {
-            if (p.decay_row && !p.s_code) cp_async16(reinterpret_cast<uint8_t*>(S.s) + 16 * c,
-                                                     reinterpret_cast<const uint8_t*>(p.s + tok * DK) + 16 * c);
-        } else if ((c -= C32) < C8) {
-            if (p.decay_row && p.s_code) cp_async16(S.scode + 16 * c, p.s_code + tok * DK + 16 * c);
-        }
-        // scalars and the offsets of the head after this one
-        const int gn = g + gridDim.x;
-        if (tid == 255) {
-            if (p.erase) cp_async4(&S.beta, p.beta + tok);
-            if (!p.decay_row && !p.s_code) cp_async4(&S.rate_h, p.s + tok);
-        }
-        if (tid == 254 && gn < wp.nheads) {
-            const int hn = gn - (gn / p.H) * p.H;
-            cp_async4(&S.nxt_in_off, p.in_head_off + gn);
-            cp_async4(&S.nxt_out_off, p.out_head_off + gn);
-            if (hn < p.H - 1) cp_async4(&S.nxt_in_end, p.in_head_off + gn + 1);
-        }
-        // payload window
-        const int align = DV == 128 ? 16 : 8;
-        const int nbytes = in_end - in_off;
-        const bool ok = in_off >= 0 && nbytes >= 0 && nbytes <= p.stage_bytes && in_off % align == 0 &&
-                        nbytes % align == 0 && static_cast<long long>(in_end) <= p.region_bytes;
-        if (tid == 0) {
-            S.in_off = in_off;
-            S.in_end = in_end;
-            S.out_off = out_off;
-            S.ok = ok ? 1 : 0;
-            // the following head's window ends at the next head's offset (copied above), or at
-            // the end of the region for the last head of a batch element
-            if (gn < wp.nheads && gn - (gn / p.H) * p.H == p.H - 1)
-                S.nxt_in_end = static_cast<int>(p.region_bytes);
-        }
-        if (ok) {
-            const uint8_t* src = p.in_payload + static_cast<size_t>(b) * p.region_bytes + in_off;
-            if (DV == 128) {
-                for (int i = tid; i < nbytes / 16; i += blockDim.x) cp_async16(pay + 16 * i, src + 16 * i);
-            } else {
-                for (int i = tid; i < nbytes / 8; i += blockDim.x) cp_async8(pay + 8 * i, src + 8 * i);
-            }
-        }
-        cp_async_commit();
+    const int b = g / p.H, h = g - (g / p.H) * p.H;
+    const size_t tok = (static_cast<size_t>(b) * T + p.t_begin) * p.H + h;
+    const size_t rb = static_cast<size_t>(g) * DK;
+    // fixed-size arrays, 16-byte chunks
+    constexpr int C8 = DK / 16, C16 = DK * 2 / 16, C32 = DK * 4 / 16, CV = DV * 4 / 16;
+    int c = tid;
+    if (c < C8) cp_async16(S.w_in + 16 * c, p.in_widths + rb + 16 * c);
+    else if ((c -= C8) < C8) cp_async16(S.w_out + 16 * c, p.out_widths + rb + 16 * c);
+    else if ((c -= C8) < C8) cp_async16(S.fidx + 16 * c, p.in_fidx + rb + 16 * c);
+    else if ((c -= C8) < C16) cp_async16(reinterpret_cast<uint8_t*>(S.sc_in) + 16 * c,
+                                         reinterpret_cast<const uint8_t*>(p.in_scales + rb) + 16 * c);
+    else if ((c -= C16) < C32) cp_async16(reinterpret_cast<uint8_t*>(S.k) + 16 * c,
+                                          reinterpret_cast<const uint8_t*>(p.k + tok * DK) + 16 * c);
+    else if ((c -= C32) < C32) cp_async16(reinterpret_cast<uint8_t*>(S.q) + 16 * c,
+                                          reinterpret_cast<const uint8_t*>(p.q + tok * DK) + 16 * c);
+    else if ((c -= C32) < CV) cp_async16(reinterpret_cast<uint8_t*>(S.v) + 16 * c,
+                                         reinterpret_cast<const uint8_t*>(p.v + tok * DV) + 16 * c);
+    else if ((c -= CV) < C32) {
+        if (stats) cp_async16(reinterpret_cast<uint8_t*>(S.ms) + 16 * c,
+                              reinterpret_cast<const uint8_t*>(p.ema_s + rb) + 16 * c);
+    } else if ((c -= C32) < C32) {
+        if (stats) cp_async16(reinterpret_cast<uint8_t*>(S.mr) + 16 * c,
+                              reinterpret_cast<const uint8_t*>(p.ema_r + rb) + 16 * c);
+    } else if ((c -= C32) < C32) {
+        if (p.decay_row && !p.s_code) cp_async16(reinterpret_cast<uint8_t*>(S.s) + 16 * c,
+                                                 reinterpret_cast<const uint8_t*>(p.s + tok * DK) + 16 * c);
+    } else if ((c -= C32) < C8) {
+        if (p.decay_row && p.s_code) cp_async16(S.scode + 16 * c, p.s_code + tok * DK + 16 * c);
     }
+    // the head's decay levels (DK x L floats, 16-byte chunks) when L <= 4
+    if (p.decay_row && p.s_code && p.L <= 4) {
+        const int nch = DK * p.L / 4;
+        const float* src = p.s_lut + static_cast<size_t>(h) * DK * p.L;
+        for (int i = tid; i < nch; i += blockDim.x) cp_async16(S.lut + 4 * i, src + 4 * i);
+    }
+    // scalars and the offsets of the next head
+    if (tid == blockDim.x - 1) {
+        if (p.erase) cp_async4(&S.beta, p.beta + tok);
+        if (!p.decay_row && !p.s_code) cp_async4(&S.rate_h, p.s + tok);
+    }
+    const bool next_last = gnext >= 0 && gnext - (gnext / p.H) * p.H == p.H - 1;
+    if (tid == blockDim.x - 2 && gnext >= 0) {
+        cp_async4(&S.nxt_in_off, p.in_head_off + gnext);
+        cp_async4(&S.nxt_out_off, p.out_head_off + gnext);
+        if (!next_last) cp_async4(&S.nxt_in_end, p.in_head_off + gnext + 1);
+    }
+    // payload window (copied by wb_issue_payload)
+    const int align = DV == 128 ? 16 : 8;
+    const int nbytes = in_end - in_off;
+    const bool ok = in_off >= 0 && nbytes >= 0 && nbytes <= p.stage_bytes && in_off % align == 0 &&
+                    nbytes % align == 0 && static_cast<long long>(in_end) <= p.region_bytes;
+    if (tid == 0) {
+        S.in_off = in_off;
+        S.in_end = in_end;
+        S.out_off = out_off;
+        S.ok = ok ? 1 : 0;
+        // the next head's window ends at the head after it (copied above), or at the end of the
+        // region for the last head of a batch element
+        if (next_last) S.nxt_in_end = static_cast<int>(p.region_bytes);
+    }
+    cp_async_commit();
+}
+
+// Copy head g's packed rows (the window recorded in S by wb_issue_meta; S.ok must be visible
+// to every thread) into pay.  One commit group per call.
+template <int DK, int DV>
+__device__ __noinline__ void wb_issue_payload(const WbStage<DK, DV>& S, uint8_t* pay, int g, const WbParams& wp) {
+    const StepParams& p = wp.s;
+    const int tid = threadIdx.x;
+    if (S.ok) {
+        const int b = g / p.H;
+        const int nbytes = S.in_end - S.in_off;
+        const uint8_t* src = p.in_payload + static_cast<size_t>(b) * p.region_bytes + S.in_off;
+        if (DV == 128) {
+            for (int i = tid; i < nbytes / 16; i += blockDim.x) cp_async16(pay + 16 * i, src + 16 * i);
+        } else {
+            for (int i = tid; i < nbytes / 8; i += blockDim.x) cp_async8(pay + 8 * i, src + 8 * i);
+        }
+    }
+    cp_async_commit();
+}
 
 // ---- the kernel ---------------------------------------------------------------------------------
 template <int DK, int DV, int NW>
-__global__ void __launch_bounds__(NW * 32, 1) wb_row_kernel(const WbParams wp) {
-    constexpr int NT = NW * 32, RPW = DK / NW, CPL = DV / 32, CP2 = CPL / 2;
-    constexpr int LOGR = RPW == 16 ? 4 : RPW == 8 ? 3 : RPW == 4 ? 2 : 1;
+__global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
+    using Geo = WbGeom<DK, DV, NW>;
+    constexpr int RPW = Geo::RPW, CPL = Geo::CPL, CP2 = CPL / 2;
+    constexpr int TPR = Geo::TPR, RPB = Geo::RPB, KPT = Geo::KPT, NB = DK / RPB;
+    static_assert(CPL == 2 || CPL == 4, "value columns");
+    static_assert(RPW >= 2 && RPW <= 16 && NW == 8, "warps");
     using Sm = WbSmem<DK, DV, NW>;
     using Stage = WbStage<DK, DV>;
-    static_assert(RPW >= 2 && RPW <= 16, "rows per warp");
     const StepParams& p = wp.s;
     extern __shared__ __align__(16) uint8_t smem_raw[];
     Sm& sm = *reinterpret_cast<Sm*>(smem_raw);
-    const int pstride = (p.stage_bytes + 32 + 15) & ~15;
-    uint8_t* pay0 = smem_raw + sizeof(Sm);
-    uint8_t* pout = pay0 + 2 * pstride;
+    uint8_t* pay = smem_raw + sizeof(Sm);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const bool stats = p.ema_s != nullptr;
     const int T = p.T;
@@ -279,30 +375,31 @@ __global__ void __launch_bounds__(NW * 32, 1) wb_row_kernel(const WbParams wp) {
         sm.wc[w] = make_float4(n, w >= 2 ? __frcp_rn(n) : 0.0f, kMagic - n, kMagic + n);
     }
 
-    const int g0 = blockIdx.x;
-    if (g0 >= wp.nheads) return;
+    // a contiguous block of heads per CTA
+    const int g_begin = static_cast<int>(static_cast<long long>(blockIdx.x) * wp.nheads / gridDim.x);
+    const int g_end = static_cast<int>(static_cast<long long>(blockIdx.x + 1) * wp.nheads / gridDim.x);
+    if (g_begin >= g_end) return;
     {
-        const int h0 = g0 % p.H;
-        const int io = static_cast<int>(p.in_head_off[g0]);
-        const int ie = h0 < p.H - 1 ? static_cast<int>(p.in_head_off[g0 + 1]) : static_cast<int>(p.region_bytes);
-        const int oo = static_cast<int>(p.out_head_off[g0]);
-        wb_issue<DK, DV>(sm.st[0], pay0, g0, io, ie, oo, wp);
+        const int h0 = g_begin % p.H;
+        const int io = static_cast<int>(p.in_head_off[g_begin]);
+        const int ie = h0 < p.H - 1 ? static_cast<int>(p.in_head_off[g_begin + 1]) : static_cast<int>(p.region_bytes);
+        const int oo = static_cast<int>(p.out_head_off[g_begin]);
+        wb_issue_meta<DK, DV>(sm.st[0], g_begin, g_begin + 1 < g_end ? g_begin + 1 : -1, io, ie, oo, wp);
+        __syncthreads();
+        wb_issue_payload<DK, DV>(sm.st[0], pay, g_begin, wp);
     }
 
-    for (int j = 0;; ++j) {
-        const int g = g0 + j * gridDim.x;
-        if (g >= wp.nheads) break;
+    for (int g = g_begin, j = 0; g < g_end; ++g, ++j) {
         const int sidx = j & 1;
         Stage& S = sm.st[sidx];
-        const uint8_t* pay = pay0 + sidx * pstride;
         const int b = g / p.H, h = g - (g / p.H) * p.H;
         cp_async_wait_all();
         if (tid == 0) sm.flag = S.ok ? 0 : 1;
         __syncthreads();                                                               // B1
-        const int gn = g + gridDim.x;
-        if (gn < wp.nheads)
-            wb_issue<DK, DV>(sm.st[sidx ^ 1], pay0 + (sidx ^ 1) * pstride, gn, S.nxt_in_off, S.nxt_in_end,
-                             S.nxt_out_off, wp);
+        const bool has_next = g + 1 < g_end;
+        if (has_next)
+            wb_issue_meta<DK, DV>(sm.st[sidx ^ 1], g + 1, g + 2 < g_end ? g + 2 : -1, S.nxt_in_off,
+                                  S.nxt_in_end, S.nxt_out_off, wp);
 
         // ---- prep ---------------------------------------------------------------------------
         const size_t tok0 = (static_cast<size_t>(b) * T + p.t_begin) * p.H + h;
@@ -313,6 +410,7 @@ __global__ void __launch_bounds__(NW * 32, 1) wb_row_kernel(const WbParams wp) {
                                       min(static_cast<int>(p.s_code[tok0]), p.L - 1))
                               : S.rate_h;
         if (warp < 2) {
+            // row byte offsets: exclusive prefix sums of w dv / 8 (warp 0 input, warp 1 output)
             const uint8_t* wa = warp == 0 ? S.w_in : S.w_out;
             int* off = warp == 0 ? sm.off_in : sm.off_out;
             constexpr int PER = DK / 32;
@@ -348,10 +446,15 @@ __global__ void __launch_bounds__(NW * 32, 1) wb_row_kernel(const WbParams wp) {
             const int i = tid - 64;
             const float kk = S.k[i];
             float rate = rate_h;
-            if (p.decay_row)
-                rate = p.s_code ? __ldg(p.s_lut + (static_cast<size_t>(h) * DK + i) * p.L +
-                                        min(static_cast<int>(S.scode[i]), p.L - 1))
-                                : S.s[i];
+            if (p.decay_row) {
+                if (p.s_code) {
+                    const int code = min(static_cast<int>(S.scode[i]), p.L - 1);
+                    rate = p.L <= 4 ? S.lut[i * p.L + code]
+                                    : __ldg(p.s_lut + (static_cast<size_t>(h) * DK + i) * p.L + code);
+                } else {
+                    rate = S.s[i];
+                }
+            }
             if (!(rate > 0.0f) || !(rate < INFINITY)) raise_status(p.status, QS_DEV_RATE);
             const float d = expf(-rate);
             if (stats) {
@@ -371,38 +474,68 @@ __global__ void __launch_bounds__(NW * 32, 1) wb_row_kernel(const WbParams wp) {
             sm.deq[i] = make_float4(-A, (w >= 2 ? D : (w == 1 ? -2.0f * D : 0.0f)) * d,
                                     (w == 1 ? D : 0.0f) * d, 0.0f);
             sm.a[i] = __fmul_rn(beta0, kk);
-        } else if (tid >= 64 + DK && tid < 128 + DK) {
-            // k . q over DK rows: 64 threads, DK / 64 rows each
-            float kq = 0.0f;
+            // k . q: one partial per warp of rows
+            const float kq = warp_sum(kk * S.q[i]);
+            if (lane == 0) sm.wsum[(tid - 64) >> 5] = kq;
+        } else if (warp == 6 || warp == 7) {
+            // rows in order of width (counting sort; any order within a width)
+            const uint8_t* wa = warp == 6 ? S.w_in : S.w_out;
+            uint8_t* ord = warp == 6 ? sm.ord_in : sm.ord_out;
+            int* cnt = sm.cnt[warp - 6];
+            if (lane < 17) cnt[lane] = 0;
+            __syncwarp();
+            constexpr int PER = DK / 32;
+            int slot[PER], wv[PER];
 #pragma unroll
-            for (int r = tid - 64 - DK; r < DK; r += 64) kq = fmaf(S.k[r], S.q[r], kq);
-            kq = warp_sum(kq);
-            if (lane == 0) sm.wsum[(tid - 64 - DK) >> 5] = kq;
+            for (int jj = 0; jj < PER; ++jj) {
+                wv[jj] = min(static_cast<int>(wa[lane * PER + jj]), 16);
+                slot[jj] = atomicAdd(&cnt[wv[jj]], 1);
+            }
+            __syncwarp();
+            const int c = lane < 17 ? cnt[lane] : 0;
+            int incl = c;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int n = __shfl_up_sync(kFull, incl, o);
+                if (lane >= o) incl += n;
+            }
+            __syncwarp();
+            if (lane < 17) cnt[lane] = incl - c;
+            __syncwarp();
+#pragma unroll
+            for (int jj = 0; jj < PER; ++jj) ord[cnt[wv[jj]] + slot[jj]] = static_cast<uint8_t>(lane * PER + jj);
         }
         __syncthreads();                                                               // B2
         if (sm.flag != 0) {
             if (tid == 0) raise_status(p.status, QS_DEV_LAYOUT);
+            if (has_next) wb_issue_payload<DK, DV>(sm.st[sidx ^ 1], pay, g + 1, wp);
             continue;
         }
 
-        // ---- unpack + dequantise (first token's decay folded in) -------------------------------
+        // ---- unpack + dequantise (row layout; first token's decay folded in) -------------------
+        for (int bat = warp; bat < NB; bat += NW) {
+            const int i = sm.ord_in[bat * RPB + lane / TPR], q = lane % TPR;
+            const int w = S.w_in[i];
+            unpack_row<DV>(w, pay + sm.off_in[i] + 4 * w * q, sm.deq[i], sm.sbuf, i, q);
+        }
+        __syncthreads();                                                               // B3
+        // the payload buffer is free: the next head's packed rows
+        if (has_next) wb_issue_payload<DK, DV>(sm.st[sidx ^ 1], pay, g + 1, wp);
+
+        // ---- tokens of the interval (Eq. 1), update layout ---------------------------------------
         float2 x[RPW][CP2];
 #pragma unroll
         for (int r = 0; r < RPW; ++r) {
             const int i = warp * RPW + r;
-            uint32_t u[CPL];
-            extract_codes<CPL>(pay + sm.off_in[i], lane, S.w_in[i], u);
-            const float4 dq = sm.deq[i];
-            const float2 A2 = make_float2(dq.x, dq.x), S2 = make_float2(dq.y, dq.y), B2 = make_float2(dq.z, dq.z);
-#pragma unroll
-            for (int c = 0; c < CP2; ++c) {
-                const float2 t = make_float2(__uint_as_float(kTwo23Bits | u[2 * c]),
-                                             __uint_as_float(kTwo23Bits | u[2 * c + 1]));
-                x[r][c] = __ffma2_rn(__fadd2_rn(t, A2), S2, B2);
+            if constexpr (CPL == 4) {
+                const float4 v = *reinterpret_cast<const float4*>(sm.sbuf + sb_off<DV>(i, lane));
+                x[r][0] = make_float2(v.x, v.y);
+                x[r][1] = make_float2(v.z, v.w);
+            } else {
+                x[r][0] = *reinterpret_cast<const float2*>(sm.sbuf + sb_off<DV>(i, lane >> 1) + 2 * (lane & 1));
             }
         }
 
-        // ---- tokens of the interval (Eq. 1) ----------------------------------------------------
         for (int t = p.t_begin; t < p.t_end; ++t) {
             const size_t tok = (static_cast<size_t>(b) * T + t) * p.H + h;
             const float* kv = S.k;
@@ -469,31 +602,27 @@ __global__ void __launch_bounds__(NW * 32, 1) wb_row_kernel(const WbParams wp) {
             }
 #pragma unroll
             for (int c = 0; c < CP2; ++c) {
-                reinterpret_cast<float2*>(&sm.red[0][warp][lane * CPL])[c] = pp[c];
-                reinterpret_cast<float2*>(&sm.red[1][warp][lane * CPL])[c] = rr[c];
+                reinterpret_cast<float2*>(&sm.rc.red[0][warp][lane * CPL])[c] = pp[c];
+                reinterpret_cast<float2*>(&sm.rc.red[1][warp][lane * CPL])[c] = rr[c];
             }
-            __syncthreads();                                                           // B3
+            __syncthreads();                                                           // B4
             if (tid < DV) {
                 const int jv = tid;
                 float P = 0.0f, Rr = 0.0f;
 #pragma unroll
                 for (int w = 0; w < NW; ++w) {
-                    P += sm.red[0][w][jv];
-                    Rr += sm.red[1][w][jv];
+                    P += sm.rc.red[0][w][jv];
+                    Rr += sm.rc.red[1][w][jv];
                 }
                 kq = 0.0f;
-                if (t > p.t_begin) {
 #pragma unroll
-                    for (int w = 0; w < DK / 32; ++w) kq += sm.wsum[w];
-                } else {
-                    kq = sm.wsum[0] + sm.wsum[1];
-                }
+                for (int w = 0; w < DK / 32; ++w) kq += sm.wsum[w];
                 const float vj = vv[jv];
                 const float uu = p.erase ? __fsub_rn(__fmul_rn(beta, vj), P) : vj;
                 sm.u[jv] = uu;
                 p.o[tok * DV + jv] = fmaf(uu, kq, Rr);
             }
-            __syncthreads();                                                           // B4
+            __syncthreads();                                                           // B5
 #pragma unroll
             for (int r = 0; r < RPW; ++r) {
                 const float ki = kv[warp * RPW + r];
@@ -504,153 +633,115 @@ __global__ void __launch_bounds__(NW * 32, 1) wb_row_kernel(const WbParams wp) {
             }
         }
 
-        // ---- write-back (warp-local until B5) ---------------------------------------------------
+        // state to the buffer
+#pragma unroll
+        for (int r = 0; r < RPW; ++r) {
+            const int i = warp * RPW + r;
+            if constexpr (CPL == 4)
+                *reinterpret_cast<float4*>(sm.sbuf + sb_off<DV>(i, lane)) =
+                    make_float4(x[r][0].x, x[r][0].y, x[r][1].x, x[r][1].y);
+            else
+                *reinterpret_cast<float2*>(sm.sbuf + sb_off<DV>(i, lane >> 1) + 2 * (lane & 1)) = x[r][0];
+        }
+        __syncthreads();                                                               // B6
+
+        // ---- write-back (row layout) ----------------------------------------------------------
         const bool refit = (p.fit_every <= 1) || ((p.w_index + h) % p.fit_every == 0);
-        // row ranges (and 1-bit sums)
-#pragma unroll
-        for (int r = 0; r < RPW; ++r) {
-            const int i = warp * RPW + r;
-            float amax = 0.0f, asum = 0.0f;
-#pragma unroll
-            for (int c = 0; c < CP2; ++c) {
-                amax = fmaxf(amax, fmaxf(fabsf(x[r][c].x), fabsf(x[r][c].y)));
-                asum += fabsf(x[r][c].x) + fabsf(x[r][c].y);
-            }
-            const float R = warp_absmax(amax);
-            if (S.w_out[i] == 1) asum = warp_sum(asum);
-            if (lane == 0) {
-                sm.rowR[i] = R;
-                sm.rowM[i] = asum;
-            }
-        }
-        __syncwarp();
-        // per-row steps (lane r <-> row r): 1-bit means, rows that keep their factor, zero rows
-        float myD = 0.0f, myInv = 0.0f;
-        if (lane < RPW) {
-            const int i = warp * RPW + lane, w = S.w_out[i];
-            const float R = sm.rowR[i];
-            int fidx = S.fidx[i];
-            if (w == 1) {
-                myD = f16_round(__fdiv_rn(sm.rowM[i], static_cast<float>(DV)));
-            } else if (w >= 2) {
-                if (R == 0.0f) {
-                    if (refit) fidx = kNFit - 1;
-                } else if (!refit) {
-                    myD = cand_step(sm.fitf[fidx], R, sm.wc[w].y);
-                    myInv = step_rcp(myD);
-                }
-            }
-            sm.out_fidx[i] = static_cast<uint8_t>(fidx);
-            sm.out_scale[i] = f16_bits(myD);
-        }
-        if (refit) {
-            // the 16 candidate steps of every row: RPW x 16 (row, candidate) pairs over 32 lanes
-#pragma unroll
-            for (int pr = lane; pr < RPW * kNFit; pr += 32) {
-                const int i = warp * RPW + (pr >> 4), k = pr & 15;
-                const int w = S.w_out[i];
-                const float R = sm.rowR[i];
-                const float Dk = (w >= 2 && R > 0.0f) ? cand_step(sm.fitf[k], R, sm.wc[w].y) : 0.0f;
-                sm.cand[i][k][0] = Dk;
-                sm.cand[i][k][1] = step_rcp(Dk);
-            }
-            __syncwarp();
-            // squared-error search: candidates outer, rows inner; lane l ends with row
-            // (l >> (5 - LOGR)) and keeps the running minimum (ties to the larger factor)
-            float2 ax[RPW][CP2];
-#pragma unroll
-            for (int r = 0; r < RPW; ++r)
-#pragma unroll
-                for (int c = 0; c < CP2; ++c) ax[r][c] = make_float2(fabsf(x[r][c].x), fabsf(x[r][c].y));
-            float bsse = INFINITY;
-            int bk = 0;
-            const float2 mg2 = make_float2(kMagic, kMagic), nmg2 = make_float2(-kMagic, -kMagic);
-#pragma unroll 1
-            for (int k = 0; k < kNFit; ++k) {
-                float part[RPW];
-#pragma unroll
-                for (int r = 0; r < RPW; ++r) {
-                    const int i = warp * RPW + r;
-                    const float2 cd = *reinterpret_cast<const float2*>(&sm.cand[i][k][0]);
-                    const float lim = sm.wc[S.w_out[i]].w;
-                    const float2 inv2 = make_float2(cd.y, cd.y), nD2 = make_float2(-cd.x, -cd.x);
-                    float2 acc = make_float2(0.0f, 0.0f);
-#pragma unroll
-                    for (int c = 0; c < CP2; ++c) {
-                        float2 t = __ffma2_rn(ax[r][c], inv2, mg2);
-                        t.x = fminf(t.x, lim);
-                        t.y = fminf(t.y, lim);
-                        const float2 e = __ffma2_rn(__fadd2_rn(t, nmg2), nD2, ax[r][c]);
-                        acc = __ffma2_rn(e, e, acc);
-                    }
-                    part[r] = acc.x + acc.y;
-                }
-                const float tot = reduce_rows<RPW>(part, lane);
-                if (tot <= bsse) {
-                    bsse = tot;
-                    bk = k;
-                }
-            }
-            if ((lane & ((32 >> LOGR) - 1)) == 0) sm.best_k[warp * RPW + (lane >> (5 - LOGR))] = bk;
-            __syncwarp();
-        }
-        // codes, folded into one 64-bit chunk per lane and row
-#pragma unroll
-        for (int r = 0; r < RPW; ++r) {
-            const int i = warp * RPW + r;
+        for (int bat = warp; bat < NB; bat += NW) {
+            const int i = sm.ord_out[bat * RPB + lane / TPR], q = lane % TPR;
             const int w = S.w_out[i];
-            float D = __shfl_sync(kFull, myD, r), inv = __shfl_sync(kFull, myInv, r);
-            uint32_t u[4] = {0u, 0u, 0u, 0u};
-            if (w >= 2) {
-                const float4 wc = sm.wc[w];
-                if (refit && sm.rowR[i] > 0.0f) {
-                    const int best = sm.best_k[i];
-                    const float2 cd = *reinterpret_cast<const float2*>(&sm.cand[i][best][0]);
-                    D = cd.x;
-                    inv = cd.y;
-                    if (lane == 0) {
-                        sm.out_fidx[i] = static_cast<uint8_t>(best);
-                        sm.out_scale[i] = f16_bits(D);
+            float2 xv[16], av[16];
+#pragma unroll
+            for (int g2 = 0; g2 < 8; ++g2) {
+                const float4 v = *reinterpret_cast<const float4*>(sm.sbuf + sb_off<DV>(i, 8 * q + g2));
+                xv[2 * g2] = make_float2(v.x, v.y);
+                xv[2 * g2 + 1] = make_float2(v.z, v.w);
+            }
+            // row range R = max |x| (identical in the row's TPR lanes)
+            float R = 0.0f;
+#pragma unroll
+            for (int c = 0; c < 16; ++c) {
+                av[c] = make_float2(fabsf(xv[c].x), fabsf(xv[c].y));
+                R = fmaxf(R, fmaxf(av[c].x, av[c].y));
+            }
+#pragma unroll
+            for (int o = 1; o < TPR; o <<= 1) R = fmaxf(R, __shfl_xor_sync(kFull, R, o));
+            float D = 0.0f;
+            int fidx = S.fidx[i];
+            if (__any_sync(kFull, w == 1)) {
+                // 1-bit rows: mean |x|
+                float2 s2 = make_float2(0.0f, 0.0f);
+#pragma unroll
+                for (int c = 0; c < 16; ++c) s2 = __fadd2_rn(s2, av[c]);
+                float sum = s2.x + s2.y;
+#pragma unroll
+                for (int o = 1; o < TPR; o <<= 1) sum += __shfl_xor_sync(kFull, sum, o);
+                if (w == 1) D = f16_round(__fdiv_rn(sum, static_cast<float>(DV)));
+            }
+            const float inv_n = sm.wc[w > 16 ? 0 : w].y;
+            if (refit) {
+                __syncwarp();   // the previous batch's rows are done with the candidate table
+                // the row's 16 candidate steps, KPT per lane.  The search takes approximate
+                // reciprocals; the chosen step's IEEE reciprocal is taken below for the codes.
+#pragma unroll
+                for (int kk = 0; kk < KPT; ++kk) {
+                    const int k = q * KPT + kk;
+                    const float Dk = (w >= 2 && R > 0.0f) ? cand_step(sm.fitf[k], R, inv_n) : 0.0f;
+                    float ik = 0.0f;
+                    if (Dk > 0.0f) asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(ik) : "f"(Dk));
+                    sm.rc.cand[warp][lane / TPR][k] = make_float2(ik, -Dk);
+                }
+                __syncwarp();
+                // squared error of every candidate (levels clamped at n): e = |x| - q Delta,
+                // q = min(rint(|x| / Delta), n).  The smallest wins; ties go to the larger factor.
+                const float lim = sm.wc[w > 16 ? 0 : w].w;
+                const float2 M2 = make_float2(kMagic, kMagic), nM2 = make_float2(-kMagic, -kMagic);
+                float bsse = INFINITY;
+                int bk = 0;
+#pragma unroll 1
+                for (int k = 0; k < kNFit; ++k) {
+                    const float2 cd = sm.rc.cand[warp][lane / TPR][k];
+                    const float2 i2 = make_float2(cd.x, cd.x), d2 = make_float2(cd.y, cd.y);
+                    float2 acc0 = make_float2(0.0f, 0.0f), acc1 = make_float2(0.0f, 0.0f);
+#pragma unroll
+                    for (int c = 0; c < 16; c += 2) {
+                        float2 t0 = __ffma2_rn(av[c], i2, M2);
+                        float2 t1 = __ffma2_rn(av[c + 1], i2, M2);
+                        t0.x = fminf(t0.x, lim);
+                        t0.y = fminf(t0.y, lim);
+                        t1.x = fminf(t1.x, lim);
+                        t1.y = fminf(t1.y, lim);
+                        const float2 e0 = __ffma2_rn(__fadd2_rn(t0, nM2), d2, av[c]);
+                        const float2 e1 = __ffma2_rn(__fadd2_rn(t1, nM2), d2, av[c + 1]);
+                        acc0 = __ffma2_rn(e0, e0, acc0);
+                        acc1 = __ffma2_rn(e1, e1, acc1);
+                    }
+                    float tot = (acc0.x + acc0.y) + (acc1.x + acc1.y);
+#pragma unroll
+                    for (int o = 1; o < TPR; o <<= 1) tot += __shfl_xor_sync(kFull, tot, o);
+                    if (tot <= bsse) {
+                        bsse = tot;
+                        bk = k;
                     }
                 }
-                const float2 inv2 = make_float2(inv, inv), mg2 = make_float2(kMagic, kMagic);
-                const uint32_t off = kMagicBits - static_cast<uint32_t>(wc.x);
-#pragma unroll
-                for (int c = 0; c < CP2; ++c) {
-                    const float2 tq = __fadd2_rn(__fmul2_rn(x[r][c], inv2), mg2);
-                    u[2 * c] = __float_as_uint(fminf(fmaxf(tq.x, wc.z), wc.w)) - off;
-                    u[2 * c + 1] = __float_as_uint(fminf(fmaxf(tq.y, wc.z), wc.w)) - off;
+                if (w >= 2) {
+                    D = -sm.rc.cand[warp][lane / TPR][bk].y;
+                    fidx = bk;
                 }
-            } else if (w == 1) {
-#pragma unroll
-                for (int c = 0; c < CP2; ++c) {
-                    u[2 * c] = x[r][c].x < 0.0f ? 1u : 0u;
-                    u[2 * c + 1] = x[r][c].y < 0.0f ? 1u : 0u;
-                }
+            } else if (w >= 2 && R > 0.0f) {
+                D = cand_step(sm.fitf[fidx], R, inv_n);
             }
-            uint64_t ch = 0;
-#pragma unroll
-            for (int c = 0; c < CPL; ++c) ch |= static_cast<uint64_t>(u[c]) << (c * w);
-            sm.chunk[warp][r][lane] = make_uint2(static_cast<uint32_t>(ch), static_cast<uint32_t>(ch >> 32));
+            if (q == 0) {
+                sm.rowR[i] = R;
+                sm.out_scale[i] = f16_bits(D);
+                sm.out_fidx[i] = static_cast<uint8_t>(fidx);
+            }
+            // codes + packed words, stored to the output region (4w bytes at byte 4 w q of the row)
+            uint8_t* orow = p.out_payload + static_cast<size_t>(b) * p.region_bytes + S.out_off + sm.off_out[i];
+            pack_row<DV == 128 ? 16 : 8>(w, xv, w >= 2 ? step_rcp(D) : 0.0f, orow + 4 * w * q);
         }
-        __syncwarp();
-#pragma unroll 1
-        for (int r = 0; r < RPW; ++r) {
-            const int i = warp * RPW + r;
-            const uint2 c2 = sm.chunk[warp][r][lane];
-            pack_row<CPL>(pout + sm.off_out[i], lane, S.w_out[i], (static_cast<uint64_t>(c2.y) << 32) | c2.x);
-        }
-        __syncthreads();                                                               // B5
+        __syncthreads();                                                               // B7
         // ---- stores -------------------------------------------------------------------------------
-        const int nbytes = sm.off_out[DK];
-        uint8_t* dst = p.out_payload + static_cast<size_t>(b) * p.region_bytes + S.out_off;
-        if (DV == 128) {
-            for (int i = tid; i < nbytes / 16; i += NT)
-                reinterpret_cast<uint4*>(dst)[i] = reinterpret_cast<const uint4*>(pout)[i];
-        } else {
-            for (int i = tid; i < nbytes / 8; i += NT)
-                reinterpret_cast<uint2*>(dst)[i] = reinterpret_cast<const uint2*>(pout)[i];
-        }
         const size_t rb = static_cast<size_t>(g) * DK;
         if (tid < DK) {
             p.out_scales[rb + tid] = sm.out_scale[tid];
@@ -672,7 +763,7 @@ cudaError_t launch_wb_row_t(const qstate_cfg& cfg, const StepParams& sp, cudaStr
     wp.s.stage_bytes = DK * DV * cfg.bmax / 8;
     wp.nheads = cfg.B * cfg.H;
     const int pstride = (wp.s.stage_bytes + 32 + 15) & ~15;
-    const size_t smem = sizeof(WbSmem<DK, DV, NW>) + 3 * static_cast<size_t>(pstride);
+    const size_t smem = sizeof(WbSmem<DK, DV, NW>) + static_cast<size_t>(pstride);
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
