@@ -8,8 +8,10 @@
 // c_i 4^{-b}: the result is the set of the M = total - N b_min most valuable bits (i, b),
 // b in (b_min, b_max].  For FP32 c the order of c 4^{-b} is the order of the integer key
 // bits(c) - b 2^24 (a power-of-4 scaling moves only the exponent field), so the kernel finds
-// the M-th largest key by bisection on integer counts -- no logarithm, no floating-point
-// comparison -- and gives bits tied at the threshold to the lowest unit indices.
+// the M-th largest key from integer counts -- no logarithm, no floating-point
+// comparison -- and gives bits tied at the threshold to the lowest unit indices.  The M-th
+// largest key is found from a histogram of the keys' high parts followed by a radix select on
+// their low 24 bits.
 #include "qs_common.cuh"
 
 namespace qs {
@@ -17,7 +19,8 @@ namespace qs {
 namespace {
 
 constexpr int kThreads = 1024;
-constexpr long long kNullKey = -73LL * (1LL << 23);   // bits of 2^-200 on a virtual exponent
+constexpr int kNullKey = -73 * (1 << 23);   // bits of 2^-200 on a virtual exponent
+constexpr int kHistOff = 64;                 // high parts -37 - 16 .. 127 -> bins 11 .. 191
 
 __device__ __forceinline__ float expm1_series(float x, const float* e1) {
     if (!(x > 0.0f)) return 0.0f;
@@ -32,31 +35,6 @@ __device__ __forceinline__ float expm1_series(float x, const float* e1) {
     float y = __fmul_rn(p, x);
     for (int i = 0; i < halvings; ++i) y = __fmul_rn(y, __fadd_rn(y, 2.0f));
     return y;
-}
-
-template <typename T>
-__device__ T block_reduce(T v, T* red, int op) {   // op 0: sum, 1: min, 2: max
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        T w = __shfl_xor_sync(kFull, v, o);
-        v = op == 0 ? v + w : (op == 1 ? (w < v ? w : v) : (w > v ? w : v));
-    }
-    __syncthreads();
-    if (lane == 0) red[warp] = v;
-    __syncthreads();
-    if (warp == 0) {
-        v = red[lane];   // blockDim.x == 1024: 32 warps
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            T w = __shfl_xor_sync(kFull, v, o);
-            v = op == 0 ? v + w : (op == 1 ? (w < v ? w : v) : (w > v ? w : v));
-        }
-        if (lane == 0) red[0] = v;
-    }
-    __syncthreads();
-    T r = red[0];
-    return r;
 }
 
 // Exclusive prefix sum over the block of one int per thread (thread order).
@@ -90,17 +68,57 @@ __device__ int block_exclusive_scan(int v, int* red, int* total) {
 
 }  // namespace
 
-__global__ void __launch_bounds__(kThreads) alloc_kernel(const AllocParams p) {
+// Warp 0 only: the bin whose suffix count (bins >= it, highest first) first reaches `rank`
+// (1-based); returns it and sets *above to the count of the bins above it.  hist has 256 bins.
+__device__ int warp_select_bin(const int* hist, int rank, int* above) {
+    const int lane = threadIdx.x & 31;
+    // lane l owns bins [8 (31 - l), 8 (31 - l) + 8): lanes in descending bin order
+    int c[8];
+    int s = 0;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        c[k] = hist[8 * (31 - lane) + 7 - k];   // descending within the lane
+        s += c[k];
+    }
+    int incl = s;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int n = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o) incl += n;
+    }
+    const int excl = incl - s;   // count of all bins above this lane's
+    const unsigned hit = __ballot_sync(kFull, excl < rank && incl >= rank);
+    const int src = __ffs(hit) - 1;
+    int bin = 0, ab = 0;
+    if (lane == src) {
+        int run = excl;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            if (run + c[k] >= rank) {
+                bin = 8 * (31 - lane) + 7 - k;
+                ab = run;
+                break;
+            }
+            run += c[k];
+        }
+    }
+    bin = __shfl_sync(kFull, bin, src);
+    *above = __shfl_sync(kFull, ab, src);
+    return bin;
+}
+
+__global__ void __launch_bounds__(kThreads, 2) alloc_kernel(const AllocParams p) {
     extern __shared__ __align__(16) uint8_t smem[];
     const int N = p.units;
-    long long* key = reinterpret_cast<long long*>(smem);
+    int* key = reinterpret_cast<int*>(smem);
     const int gsz = p.group_heads * p.dk;
     const int ngroups = p.unit_row ? N / gsz : 0;
     float* Rs = reinterpret_cast<float*>(key + N);                   // row unit: ranges
     float* gmean = Rs + (p.unit_row ? N : 0);
-    long long* redl = reinterpret_cast<long long*>(gmean + ((ngroups + 3) & ~3));
-    int* redi = reinterpret_cast<int*>(redl + 32);
-    uint8_t* wv = reinterpret_cast<uint8_t*>(redi + 72);
+    int* hist = reinterpret_cast<int*>(gmean + ((ngroups + 3) & ~3));
+    int* redi = hist + 256;
+    int* sel = redi + 72;                                              // H*, rank, low prefix
+    uint8_t* wv = reinterpret_cast<uint8_t*>(sel + 4);
     const int tid = threadIdx.x;
     const size_t base = static_cast<size_t>(blockIdx.x) * N;
 
@@ -116,10 +134,14 @@ __global__ void __launch_bounds__(kThreads) alloc_kernel(const AllocParams p) {
             gmean[g] = __fdiv_rn(acc, static_cast<float>(gsz));
         }
     }
+    for (int k = tid; k < 256; k += kThreads) hist[k] = 0;
     __syncthreads();
 
-    // 2. weights (Eq. 3) -> integer keys
-    long long kmin = LLONG_MAX, kmax = LLONG_MIN;
+    // 2. weights (Eq. 3) -> integer keys; the keys of unit u's bits b_min + j (j = 1..J) are
+    //    key_u - j 2^24, i.e. high part (key_u >> 24) - j and low part key_u & 0xFFFFFF, so every
+    //    unit adds one to a contiguous range of high parts: a difference array on 256 bins
+    const int J = p.bmax - p.bmin;
+    const long long M = p.total - static_cast<long long>(N) * p.bmin;
     for (int u = tid; u < N; u += kThreads) {
         float c = 1.0f;
         if (!p.uniform) {
@@ -136,32 +158,75 @@ __global__ void __launch_bounds__(kThreads) alloc_kernel(const AllocParams p) {
             c = __fmul_rn(G, rt2);
         }
         if (c > 0x1p60f) c = 0x1p60f;
-        const long long k = (c >= 0x1p-60f) ? static_cast<long long>(__float_as_int(c)) : kNullKey;
+        const int k = (c >= 0x1p-60f) ? __float_as_int(c) : kNullKey;
         key[u] = k;
-        kmin = k < kmin ? k : kmin;
-        kmax = k > kmax ? k : kmax;
+        if (J > 0) {
+            const int E = k >> 24;   // in [-37, 127]
+            atomicAdd(&hist[E - J + kHistOff], 1);
+            atomicAdd(&hist[E + kHistOff], -1);
+        }
     }
-    kmin = block_reduce<long long>(kmin, redl, 1);
-    kmax = block_reduce<long long>(kmax, redl, 2);
+    __syncthreads();
 
-    // 3. the M-th most valuable bit: largest T with #{(u, j): key_u - j 2^24 >= T} >= M
-    const int J = p.bmax - p.bmin;
-    const long long M = p.total - static_cast<long long>(N) * p.bmin;
+    // 3. V = the M-th largest key: its high part from the bins (prefix of the difference
+    //    array), then its low 24 bits by a radix select (8 bits per pass) over the units whose
+    //    key range covers that high part
     long long V = LLONG_MAX;   // M == 0: nothing above b_min
     if (M > 0) {
-        long long lo = kmin - static_cast<long long>(J) * (1LL << 24);   // count(lo) = N J >= M
-        long long hi = kmax - (1LL << 24) + 1;                          // count(hi) = 0 < M
-        while (hi - lo > 1) {
-            const long long mid = lo + (hi - lo) / 2;
-            int cnt = 0;
-            for (int u = tid; u < N; u += kThreads) {
-                const long long d = key[u] - mid;
-                if (d >= 0) cnt += static_cast<int>(min(d >> 24, static_cast<long long>(J)));
+        if (tid < 32) {
+            // prefix sum over 256 bins -> counts per high part
+            int c[8];
+            int s = 0;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                s += hist[8 * tid + k];
+                c[k] = s;
             }
-            cnt = block_reduce<int>(cnt, redi, 0);
-            if (cnt >= M) lo = mid; else hi = mid;
+            int incl = s;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int n = __shfl_up_sync(kFull, incl, o);
+                if (tid >= o) incl += n;
+            }
+            const int ex = incl - s;
+            __syncwarp();
+#pragma unroll
+            for (int k = 0; k < 8; ++k) hist[8 * tid + k] = ex + c[k];
+            __syncwarp();
+            int above = 0;
+            const int hb = warp_select_bin(hist, static_cast<int>(M), &above);
+            if (tid == 0) {
+                sel[0] = hb - kHistOff;                  // high part of V
+                sel[1] = static_cast<int>(M) - above;    // rank of V among that bin's keys
+                sel[2] = 0;                              // low bits found so far
+            }
         }
-        V = lo;
+        __syncthreads();
+        const int Hs = sel[0];
+#pragma unroll 1
+        for (int pass = 0; pass < 3; ++pass) {
+            const int sh = 16 - 8 * pass;
+            const int pre = sel[2];
+            const int pmask = pass == 0 ? 0 : (0xFFFFFF << (sh + 8)) & 0xFFFFFF;
+            for (int k = tid; k < 256; k += kThreads) hist[k] = 0;
+            __syncthreads();
+            for (int u = tid; u < N; u += kThreads) {
+                const int k = key[u];
+                const int E = k >> 24, L = k & 0xFFFFFF;
+                if (E - J <= Hs && Hs <= E - 1 && (L & pmask) == pre) atomicAdd(&hist[(L >> sh) & 255], 1);
+            }
+            __syncthreads();
+            if (tid < 32) {
+                int above = 0;
+                const int d = warp_select_bin(hist, sel[1], &above);
+                if (tid == 0) {
+                    sel[1] -= above;
+                    sel[2] = pre | (d << sh);
+                }
+            }
+            __syncthreads();
+        }
+        V = static_cast<long long>(Hs) * (1LL << 24) + sel[2];
     }
 
     // 4. widths: bits strictly above V, plus tied bits to the lowest unit indices
@@ -171,7 +236,7 @@ __global__ void __launch_bounds__(kThreads) alloc_kernel(const AllocParams p) {
     for (int u = u0; u < u1; ++u) {
         int gt = 0, tie = 0;
         if (M > 0) {
-            const long long d = key[u] - V;
+            const long long d = static_cast<long long>(key[u]) - V;
             if (d > 0) {
                 gt = static_cast<int>(min((d - 1) >> 24, static_cast<long long>(J)));
                 tie = ((d & 0xFFFFFF) == 0 && (d >> 24) <= J) ? 1 : 0;
@@ -181,13 +246,14 @@ __global__ void __launch_bounds__(kThreads) alloc_kernel(const AllocParams p) {
         gt_local += gt;
         tie_local += tie;
     }
-    const int gt_total = block_reduce<int>(gt_local, redi, 0);
+    int gt_total = 0;
+    (void)block_exclusive_scan(gt_local, redi, &gt_total);
     const long long need = M - gt_total;
     int tie_total = 0;
     int tie_before = block_exclusive_scan(tie_local, redi, &tie_total);
     for (int u = u0; u < u1; ++u) {
         if (M > 0) {
-            const long long d = key[u] - V;
+            const long long d = static_cast<long long>(key[u]) - V;
             if (d > 0 && (d & 0xFFFFFF) == 0 && (d >> 24) <= J) {
                 if (tie_before < need) wv[u] += 1;
                 ++tie_before;
@@ -210,13 +276,13 @@ __global__ void __launch_bounds__(kThreads) alloc_kernel(const AllocParams p) {
     int total_bytes = 0;
     const int off = block_exclusive_scan(tid < p.H ? hb : 0, redi, &total_bytes);
     if (tid < p.H) p.head_off[static_cast<size_t>(blockIdx.x) * p.H + tid] = static_cast<uint32_t>(off);
-    if (tid == 0 && (need < 0 || need > tie_total)) raise_status(p.status, QS_DEV_LAYOUT);
+    if (tid == 0 && M > 0 && (need < 1 || need > tie_total)) raise_status(p.status, QS_DEV_LAYOUT);
 }
 
 cudaError_t launch_alloc(const AllocParams& p, cudaStream_t stream) {
     const int ngroups = p.unit_row ? p.units / (p.group_heads * p.dk) : 0;
-    const size_t smem = static_cast<size_t>(p.units) * 8 + (p.unit_row ? p.units * 4 : 0) +
-                        ((ngroups + 3) & ~3) * 4 + 32 * 8 + 72 * 4 + p.units + 16;
+    const size_t smem = static_cast<size_t>(p.units) * 4 + (p.unit_row ? p.units * 4 : 0) +
+                        ((ngroups + 3) & ~3) * 4 + 256 * 4 + 72 * 4 + 4 * 4 + p.units + 16;
     cudaError_t e = cudaFuncSetAttribute(alloc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
