@@ -70,7 +70,8 @@ struct alignas(16) WbSmem {
     float sbuf[DK * DV];                  // FP32 state of the head (swizzled rows)
     union {
         float red[2][NW][DV];             // p and r partials per warp (token phase)
-        float2 cand[NW][32 / (DV / 32)][kNFit];   // per warp and row: (1/Delta_k, -Delta_k)
+        float2 cand[NW][32 / (DV / 32)][kNFit + 1];   // per warp and row: (1/Delta_k, -Delta_k)
+                                                      // (rows padded against bank conflicts)
     } rc;
     float4 deq[DK];                       // (-A, S, B, 0): x = (2^23 + u - A) S + B
     float4 wc[17];                        // per width: (n, 1/n, 2^23*1.5 - n, 2^23*1.5 + n)
@@ -658,12 +659,13 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                 xv[2 * g2 + 1] = make_float2(v.z, v.w);
             }
             // row range R = max |x| (identical in the row's TPR lanes)
-            float R = 0.0f;
+            float lmax = 0.0f;
 #pragma unroll
             for (int c = 0; c < 16; ++c) {
                 av[c] = make_float2(fabsf(xv[c].x), fabsf(xv[c].y));
-                R = fmaxf(R, fmaxf(av[c].x, av[c].y));
+                lmax = fmaxf(lmax, fmaxf(av[c].x, av[c].y));
             }
+            float R = lmax;
 #pragma unroll
             for (int o = 1; o < TPR; o <<= 1) R = fmaxf(R, __shfl_xor_sync(kFull, R, o));
             float D = 0.0f;
@@ -692,15 +694,32 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                     sm.rc.cand[warp][lane / TPR][k] = make_float2(ik, -Dk);
                 }
                 __syncwarp();
-                // squared error of every candidate (levels clamped at n): e = |x| - q Delta,
-                // q = min(rint(|x| / Delta), n).  The smallest wins; ties go to the larger factor.
-                const float lim = sm.wc[w > 16 ? 0 : w].w;
+                // squared error of the candidates (levels clamped at n): e = |x| - q Delta,
+                // q = min(rint(|x| / Delta), n); the smallest wins, ties to the larger factor.
+                // Candidates are taken from the largest factor down.  Every element at or above
+                // n Delta_k quantises to n, so the clipping error of the lanes' maxima is a lower
+                // bound on candidate k's error that grows as k falls: once it exceeds the best
+                // error found (with a 2^-10 margin for rounding), no smaller factor can win.
+                const float lim = sm.wc[w > 16 ? 0 : w].w, nf = sm.wc[w > 16 ? 0 : w].x;
+                float mx[TPR];
+#pragma unroll
+                for (int jl = 0; jl < TPR; ++jl) mx[jl] = __shfl_sync(kFull, lmax, (lane & ~(TPR - 1)) + jl);
                 const float2 M2 = make_float2(kMagic, kMagic), nM2 = make_float2(-kMagic, -kMagic);
+                const float2* crow = sm.rc.cand[warp][lane / TPR];
                 float bsse = INFINITY;
-                int bk = 0;
+                int bk = kNFit - 1;
 #pragma unroll 1
-                for (int k = 0; k < kNFit; ++k) {
-                    const float2 cd = sm.rc.cand[warp][lane / TPR][k];
+                for (int k = kNFit - 1; k >= 0; --k) {
+                    const float2 cd = crow[k];
+                    const float Lk = -nf * cd.y;
+                    float lb = 0.0f;
+#pragma unroll
+                    for (int jl = 0; jl < TPR; ++jl) {
+                        const float e = fmaxf(mx[jl] - Lk, 0.0f);
+                        lb = fmaf(e, e, lb);
+                    }
+                    const bool go = w >= 2 && lb <= bsse * (1.0f + 1.0f / 1024.0f);
+                    if (!__any_sync(kFull, go)) break;
                     const float2 i2 = make_float2(cd.x, cd.x), d2 = make_float2(cd.y, cd.y);
                     float2 acc0 = make_float2(0.0f, 0.0f), acc1 = make_float2(0.0f, 0.0f);
 #pragma unroll
@@ -719,7 +738,7 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                     float tot = (acc0.x + acc0.y) + (acc1.x + acc1.y);
 #pragma unroll
                     for (int o = 1; o < TPR; o <<= 1) tot += __shfl_xor_sync(kFull, tot, o);
-                    if (tot <= bsse) {
+                    if (go && tot < bsse) {
                         bsse = tot;
                         bk = k;
                     }
