@@ -7,28 +7,31 @@
 // other's work) walks a contiguous block of heads.  While it works on head g, cp.async copies
 // head g + 1's metadata into the other half of a double buffer (widths in/out, FP16 scales,
 // fitted-factor indices, EMA statistics, the first token's k, q, v, rates and their level table)
-// and, once head g is unpacked, head g + 1's packed rows into the single payload buffer (their
-// byte window comes from offsets fetched one head earlier).
+// and, once head g's tokens are done, head g + 1's packed rows into the single payload buffer
+// (their byte window comes from offsets fetched one head earlier).
 //
-// Two thread layouts share the head's FP32 state through a shared-memory buffer (16-byte
-// groups XOR-swizzled per row):
-//  * row layout: TPR = dv/32 lanes per row, each owning 32 consecutive value columns, i.e. a
-//    word-aligned run of 32 codes (4w bytes).  Warps take rows in order of width (a counting
-//    sort per head), so the code arithmetic of a warp is specialised for one width.  Used to
-//    unpack + dequantise and for the write-back (range, factor search, codes, packing).
+// Two thread layouts share the head's FP32 state:
 //  * update layout: warp w owns key rows [w RPW, (w+1) RPW), lane l the value columns
-//    [l CPL, (l+1) CPL), so the reductions of Eq. (1) over key rows stay in registers.
-// Per head there are seven CTA barriers:
-//   B1  the head's inputs have landed            -> issue the next head's copies
-//   B2  prep: row offsets (prefix sums of widths), rows sorted by width, layout checks,
-//       per-row decay, EMA update, dequantisation constants with the first token's decay
-//       folded in, erase vector, k.q                -> unpack (row layout) into the buffer
-//   B3  -> registers (update layout); partials p = a^T S', r = q^T S'
-//   B4  -> u = beta v - p, o = r + u (k.q)
-//   B5  -> S = S' + k u^T (further tokens of the interval repeat B3..B5), state to the buffer
-//   B6  -> write-back (row layout): row range R, the 16 candidate steps and their squared
+//    [l CPL, (l+1) CPL), so the reductions of Eq. (1) over key rows stay in registers.  The
+//    packed rows are decoded straight into it (each lane reads its CPL codes at bit
+//    l CPL w of the row, for any width w).
+//  * row layout: TPR = dv/32 lanes per row, each owning 32 consecutive value columns, i.e. a
+//    word-aligned run of 32 codes (4w bytes).  Warps take rows in order of output width (a
+//    counting sort per head), so the code arithmetic of a warp is specialised for one width.
+//    Used for the write-back (range, factor search, codes, packing); the state reaches it
+//    through a shared-memory buffer (16-byte groups XOR-swizzled per row).
+// Per head there are six CTA barriers:
+//   B1  the head's inputs have landed            -> issue the next head's metadata copies
+//   B2  prep: row offsets (prefix sums of widths), rows sorted by output width, layout
+//       checks, per-row decay, EMA update, dequantisation constants with the first token's
+//       decay folded in, erase vector, k.q         -> unpack into registers (update layout),
+//       partials p = a^T S', r = q^T S'
+//   B3  -> u = beta v - p, o = r + u (k.q)
+//   B4  -> S = S' + k u^T (further tokens of the interval repeat B3..B4); the next head's
+//       packed rows are copied; state to the buffer
+//   B5  -> write-back (row layout): row range R, the 16 candidate steps and their squared
 //       errors (refit), codes, and each lane's packed words stored to the output region
-//   B7  -> coalesced stores of scales, factor indices, ranges and EMAs.
+//   B6  -> coalesced stores of scales, factor indices, ranges and EMAs.
 // The next head's B1 orders the reuse of stage and staging buffers.
 #pragma once
 
@@ -81,9 +84,10 @@ struct alignas(16) WbSmem {
     float rowR[DK];
     float fitf[kNFit];
     float wsum[NW];
-    int off_in[DK + 1], off_out[DK + 1];
-    int cnt[2][17];
-    uint8_t ord_in[DK], ord_out[DK];      // rows in order of input / output width
+    alignas(16) int off_in[DK + 4];
+    alignas(16) int off_out[DK + 4];
+    int cnt[1][17];
+    uint8_t ord_out[DK];                  // rows in order of output width
     uint16_t out_scale[DK];
     uint8_t out_fidx[DK];
     int flag;
@@ -478,11 +482,11 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
             // k . q: one partial per warp of rows
             const float kq = warp_sum(kk * S.q[i]);
             if (lane == 0) sm.wsum[(tid - 64) >> 5] = kq;
-        } else if (warp == 6 || warp == 7) {
-            // rows in order of width (counting sort; any order within a width)
-            const uint8_t* wa = warp == 6 ? S.w_in : S.w_out;
-            uint8_t* ord = warp == 6 ? sm.ord_in : sm.ord_out;
-            int* cnt = sm.cnt[warp - 6];
+        } else if (warp == 6) {
+            // rows in order of output width (counting sort; any order within a width)
+            const uint8_t* wa = S.w_out;
+            uint8_t* ord = sm.ord_out;
+            int* cnt = sm.cnt[0];
             if (lane < 17) cnt[lane] = 0;
             __syncwarp();
             constexpr int PER = DK / 32;
@@ -513,30 +517,31 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
             continue;
         }
 
-        // ---- unpack + dequantise (row layout; first token's decay folded in) -------------------
-        for (int bat = warp; bat < NB; bat += NW) {
-            const int i = sm.ord_in[bat * RPB + lane / TPR], q = lane % TPR;
-            const int w = S.w_in[i];
-            unpack_row<DV>(w, pay + sm.off_in[i] + 4 * w * q, sm.deq[i], sm.sbuf, i, q);
-        }
-        __syncthreads();                                                               // B3
-        // the payload buffer is free: the next head's packed rows
-        if (has_next) wb_issue_payload<DK, DV>(sm.st[sidx ^ 1], pay, g + 1, wp);
-
-        // ---- tokens of the interval (Eq. 1), update layout ---------------------------------------
+        // ---- unpack + dequantise into the update layout (first token's decay folded in) -------
         float2 x[RPW][CP2];
 #pragma unroll
-        for (int r = 0; r < RPW; ++r) {
-            const int i = warp * RPW + r;
-            if constexpr (CPL == 4) {
-                const float4 v = *reinterpret_cast<const float4*>(sm.sbuf + sb_off<DV>(i, lane));
-                x[r][0] = make_float2(v.x, v.y);
-                x[r][1] = make_float2(v.z, v.w);
-            } else {
-                x[r][0] = *reinterpret_cast<const float2*>(sm.sbuf + sb_off<DV>(i, lane >> 1) + 2 * (lane & 1));
+        for (int r4 = 0; r4 < RPW; r4 += 4) {
+            const int i0 = warp * RPW + r4;
+            const int4 o4 = *reinterpret_cast<const int4*>(&sm.off_in[i0]);
+            const uint32_t w4 = *reinterpret_cast<const uint32_t*>(&S.w_in[i0]);
+            const int offs[4] = {o4.x, o4.y, o4.z, o4.w};
+#pragma unroll
+            for (int rr = 0; rr < 4; ++rr) {
+                const int r = r4 + rr;
+                uint32_t u[CPL];
+                extract_codes<CPL>(pay + offs[rr], lane, static_cast<int>((w4 >> (8 * rr)) & 0xFFu), u);
+                const float4 dq = sm.deq[i0 + rr];
+                const float2 A2 = make_float2(dq.x, dq.x), S2 = make_float2(dq.y, dq.y), B2 = make_float2(dq.z, dq.z);
+#pragma unroll
+                for (int c = 0; c < CP2; ++c) {
+                    const float2 t2 = make_float2(__uint_as_float(kTwo23Bits | u[2 * c]),
+                                                  __uint_as_float(kTwo23Bits | u[2 * c + 1]));
+                    x[r][c] = __ffma2_rn(__fadd2_rn(t2, A2), S2, B2);
+                }
             }
         }
 
+        // ---- tokens of the interval (Eq. 1) ----------------------------------------------------
         for (int t = p.t_begin; t < p.t_end; ++t) {
             const size_t tok = (static_cast<size_t>(b) * T + t) * p.H + h;
             const float* kv = S.k;
@@ -591,14 +596,18 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
 #pragma unroll
             for (int c = 0; c < CP2; ++c) pp[c] = rr[c] = make_float2(0.0f, 0.0f);
 #pragma unroll
-            for (int r = 0; r < RPW; ++r) {
-                const int i = warp * RPW + r;
-                const float2 a2 = make_float2(sm.a[i], sm.a[i]);
-                const float2 q2 = make_float2(qv[i], qv[i]);
+            for (int r4 = 0; r4 < RPW; r4 += 4) {
+                const float4 a4 = *reinterpret_cast<const float4*>(&sm.a[warp * RPW + r4]);
+                const float4 q4 = *reinterpret_cast<const float4*>(&qv[warp * RPW + r4]);
+                const float as[4] = {a4.x, a4.y, a4.z, a4.w}, qs[4] = {q4.x, q4.y, q4.z, q4.w};
 #pragma unroll
-                for (int c = 0; c < CP2; ++c) {
-                    pp[c] = __ffma2_rn(x[r][c], a2, pp[c]);
-                    rr[c] = __ffma2_rn(x[r][c], q2, rr[c]);
+                for (int j4 = 0; j4 < 4; ++j4) {
+                    const float2 a2 = make_float2(as[j4], as[j4]), q2 = make_float2(qs[j4], qs[j4]);
+#pragma unroll
+                    for (int c = 0; c < CP2; ++c) {
+                        pp[c] = __ffma2_rn(x[r4 + j4][c], a2, pp[c]);
+                        rr[c] = __ffma2_rn(x[r4 + j4][c], q2, rr[c]);
+                    }
                 }
             }
 #pragma unroll
@@ -606,7 +615,7 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                 reinterpret_cast<float2*>(&sm.rc.red[0][warp][lane * CPL])[c] = pp[c];
                 reinterpret_cast<float2*>(&sm.rc.red[1][warp][lane * CPL])[c] = rr[c];
             }
-            __syncthreads();                                                           // B4
+            __syncthreads();                                                           // B3
             if (tid < DV) {
                 const int jv = tid;
                 float P = 0.0f, Rr = 0.0f;
@@ -623,17 +632,25 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                 sm.u[jv] = uu;
                 p.o[tok * DV + jv] = fmaf(uu, kq, Rr);
             }
-            __syncthreads();                                                           // B5
+            __syncthreads();                                                           // B4
+            float2 u2[CP2];
 #pragma unroll
-            for (int r = 0; r < RPW; ++r) {
-                const float ki = kv[warp * RPW + r];
-                const float2 k2 = make_float2(ki, ki);
+            for (int c = 0; c < CP2; ++c) u2[c] = reinterpret_cast<const float2*>(&sm.u[lane * CPL])[c];
 #pragma unroll
-                for (int c = 0; c < CP2; ++c)
-                    x[r][c] = __ffma2_rn(k2, reinterpret_cast<const float2*>(&sm.u[lane * CPL])[c], x[r][c]);
+            for (int r4 = 0; r4 < RPW; r4 += 4) {
+                const float4 k4 = *reinterpret_cast<const float4*>(&kv[warp * RPW + r4]);
+                const float ks[4] = {k4.x, k4.y, k4.z, k4.w};
+#pragma unroll
+                for (int j4 = 0; j4 < 4; ++j4) {
+                    const float2 k2 = make_float2(ks[j4], ks[j4]);
+#pragma unroll
+                    for (int c = 0; c < CP2; ++c) x[r4 + j4][c] = __ffma2_rn(k2, u2[c], x[r4 + j4][c]);
+                }
             }
         }
 
+        // the payload buffer is free: the next head's packed rows
+        if (has_next) wb_issue_payload<DK, DV>(sm.st[sidx ^ 1], pay, g + 1, wp);
         // state to the buffer
 #pragma unroll
         for (int r = 0; r < RPW; ++r) {
@@ -644,7 +661,7 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
             else
                 *reinterpret_cast<float2*>(sm.sbuf + sb_off<DV>(i, lane >> 1) + 2 * (lane & 1)) = x[r][0];
         }
-        __syncthreads();                                                               // B6
+        __syncthreads();                                                               // B5
 
         // ---- write-back (row layout) ----------------------------------------------------------
         const bool refit = (p.fit_every <= 1) || ((p.w_index + h) % p.fit_every == 0);
@@ -759,7 +776,7 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
             uint8_t* orow = p.out_payload + static_cast<size_t>(b) * p.region_bytes + S.out_off + sm.off_out[i];
             pack_row<DV == 128 ? 16 : 8>(w, xv, w >= 2 ? step_rcp(D) : 0.0f, orow + 4 * w * q);
         }
-        __syncthreads();                                                               // B7
+        __syncthreads();                                                               // B6
         // ---- stores -------------------------------------------------------------------------------
         const size_t rb = static_cast<size_t>(g) * DK;
         if (tid < DK) {
