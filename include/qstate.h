@@ -50,7 +50,23 @@ extern "C" {
 #define QSTATE_ERASE_NONE 1  /* a = 0, w = 1 (Eq. 1, Mamba-2)                                  */
 #define QSTATE_UNIT_ROW 0    /* width + FP16 scale per row (Sec. 3, "Allocation units")       */
 #define QSTATE_UNIT_HEAD 1   /* width per head, FP16 scale per 32 key rows x value column     */
-#define QSTATE_WEIGHT_OURS 0 /* c_i = Gamma_hat_i Rtilde_i^2 (Eq. 3)                           */
+/* Allocation weights c_i (Eq. 3 and the alternatives of Table 1).  With the EMAs of
+ * qstate_stats, m_s = EMA(1 - e^{-2s}) and m_r = EMA of the erasure term:
+ * Gamma_hat = (1 - m_s) / (expm1(m_r) + m_s); Rtilde^2 = R^2 / mean of R^2 over the unit's
+ * output-normalisation group (1 for the head unit, which has no per-unit range, as R is). */
+#define QSTATE_WEIGHT_OURS 0      /* Gamma_hat Rtilde^2 (Eq. 3)                                  */
+#define QSTATE_WEIGHT_RANGE 1     /* R^2, range alone                                            */
+#define QSTATE_WEIGHT_GAMMA_RAW 2 /* Gamma_hat R^2, raw range                                    */
+#define QSTATE_WEIGHT_NRANGE 3    /* Rtilde^2, relative range                                    */
+#define QSTATE_WEIGHT_PERSIST 4   /* w1 Rtilde^2, persistence w1 = 1/(1 - e^{-2s}) = 1 / m_s      */
+#define QSTATE_WEIGHT_WBFACTOR 5  /* h Rtilde^2, write-back factor h = 1/(1 - e^{-2Cs})
+                                     = 1 / (1 - (1 - m_s)^C), the power by repeated squaring    */
+#define QSTATE_WEIGHT_NOERASE 6   /* Gamma_hat with m_r = 0, times Rtilde^2                      */
+#define QSTATE_WEIGHT_SHUFFLE 7   /* Gamma_hat of unit pi(i), times Rtilde_i^2: decay weights
+                                     moved to other units by the fixed bijection
+                                     pi(i) = (A i + N/3) mod N of the batch element's N units,
+                                     A the smallest integer > 0.6180339887 N coprime to N      */
+#define QSTATE_WEIGHT_UNIFORM 8   /* equal weights: uniform widths                               */
 
 /* Method configuration.  Sizes: dk in {64, 128}, dv in {64, 128}; dk a multiple of 32 for the
  * head unit; the budget H*dk*dv*bbar must be a whole number of bytes per batch element. */
@@ -69,7 +85,7 @@ typedef struct qstate_cfg {
                                     otherwise reuses its stored factor                       */
     float ema_span;              /* EMA span in tokens (Sec. 3: 64)                           */
     int32_t gate_bits;           /* 0: FP32 decay rates; g in 1..8: log-quantised rates       */
-    int32_t weight_kind;         /* QSTATE_WEIGHT_OURS                                       */
+    int32_t weight_kind;         /* QSTATE_WEIGHT_*                                          */
 } qstate_cfg;
 
 /* One packed state (device pointers).  Layout (Sec. 3, "Levels and storage"; bit order is

@@ -115,6 +115,7 @@ def lib():
         L.orc_pack.argtypes = [ct.POINTER(OrcCfg)] + [P] * 7
         L.orc_unpack.argtypes = [ct.POINTER(OrcCfg)] + [P] * 5
         L.orc_weights.argtypes = [ct.POINTER(OrcCfg), ct.c_int, P, P, P, P]
+        L.orc_shuffle.argtypes = [ct.c_int, ct.POINTER(ct.c_int), ct.POINTER(ct.c_int)]
         L.orc_alloc_from_weights.argtypes = [ct.c_int, P, ct.c_int, ct.c_int, ct.c_long,
                                              ct.c_int, ct.c_int, P]
         L.orc_alloc.argtypes = [ct.POINTER(OrcCfg), P, P, P, P, P]
@@ -256,8 +257,15 @@ def weights(cfg: Cfg, ema_s, ema_r, rng, b=0):
     c = cfg.c()
     out = np.zeros(cfg.units, np.float32)
     args = [_c(ema_s, np.float32), _c(ema_r, np.float32), _c(rng, np.float32)]
-    lib().orc_weights(ct.byref(c), b, *[_p(a) for a in args], _p(out))
+    _check(lib().orc_weights(ct.byref(c), b, *[_p(a) for a in args], _p(out)), "weights")
     return np.where(out < 0, 0.0, out).astype(np.float32)
+
+
+def shuffle_map(N):
+    """The shuffled-decay bijection of N units (weight kind 7): u -> (A u + B) mod N."""
+    A, B = ct.c_int(), ct.c_int()
+    lib().orc_shuffle(N, ct.byref(A), ct.byref(B))
+    return (A.value * np.arange(N, dtype=np.int64) + B.value) % N
 
 
 def alloc_from_weights(cw, bmin, bmax, total, bbar_num=None, bbar_den=1):

@@ -438,11 +438,57 @@ int orc_unpack(const orc_cfg* c, const uint8_t* payload, const uint16_t* scales,
  * Weights below 2^-60 (and NaN) become the null weight 2^-200; weights above 2^60 are
  * clamped to 2^60.
  * ------------------------------------------------------------------------------------- */
+/* Table 1 replaces c_i by other weights; weight_kind selects one (0 is Eq. 3):
+ *   1  R^2                     range alone
+ *   2  Gamma_hat R^2           raw range
+ *   3  Rtilde^2                relative range
+ *   4  w1 Rtilde^2             persistence w1 = 1/(1 - e^{-2 s_hat}) = 1/m_s
+ *   5  h Rtilde^2              write-back factor h = 1/(1 - e^{-2 C s_hat}) = 1/(1 - (1 - m_s)^C),
+ *                              the power by repeated squaring (low bit of C first)
+ *   6  Gamma_hat(m_r = 0) Rtilde^2   erasure left out
+ *   7  Gamma_hat_{pi(i)} Rtilde_i^2  decay weights moved to other units by the bijection
+ *                              pi(i) = (A i + N/3) mod N, A the smallest integer > 0.6180339887 N
+ *                              coprime to N (N units per batch element)
+ *   8  1                        uniform widths
+ * The head unit has no per-unit range: R = Rtilde = 1 there. */
+static int orc_gcd(int a, int b) { return b == 0 ? a : orc_gcd(b, a % b); }
+
+void orc_shuffle(int N, int* A, int* B0) {
+    int a = (int)(0.6180339887 * N) + 1;
+    while (orc_gcd(a, N) != 1) a++;
+    *A = a % N;
+    *B0 = N / 3;
+}
+
+static float weight_of(const orc_cfg* c, int kind, float ms, float mr, float R2, float rt2) {
+    if (kind == 1) return R2;
+    if (kind == 3) return rt2;
+    if (kind == 8) return 1.0f;
+    if (kind == 4) return (1.0f / ms) * rt2;
+    if (kind == 5) {
+        float pw = 1.0f, bb = 1.0f - ms;
+        for (int e = c->C; e > 0; e >>= 1) {
+            if (e & 1) pw = pw * bb;
+            bb = bb * bb;
+        }
+        return (1.0f / (1.0f - pw)) * rt2;
+    }
+    if (kind == 6) mr = 0.0f;
+    if (mr < 0.0f) mr = 0.0f;
+    float G = (1.0f - ms) / (orc_expm1_series(mr) + ms);
+    if (kind == 2) return G * R2;
+    return G * rt2;   /* 0, 6, 7 */
+}
+
 int orc_weights(const orc_cfg* c, int b, const float* ema_s, const float* ema_r,
                 const float* range, float* cw) {
     int N = (c->unit_kind == 0) ? c->H * c->dk : c->H;
     size_t base = (size_t)b * N;
     int gsz = c->group_heads * c->dk;
+    int kind = c->weight_kind;
+    if (kind < 0 || kind > 8) return ORC_EINVAL;
+    int A = 0, B0 = 0;
+    orc_shuffle(N, &A, &B0);
     float mean = 0.0f;
     for (int u = 0; u < N; u++) {
         if (c->unit_kind == 0 && u % gsz == 0) {   /* mean R^2 of the group starting here */
@@ -450,13 +496,13 @@ int orc_weights(const orc_cfg* c, int b, const float* ema_s, const float* ema_r,
             for (int r = u; r < u + gsz; r++) acc = acc + range[base + r] * range[base + r];
             mean = acc / (float)gsz;
         }
-        float ms = ema_s[base + u];
-        float mr = ema_r[base + u];
-        if (mr < 0.0f) mr = 0.0f;
-        float G = (1.0f - ms) / (orc_expm1_series(mr) + ms);
-        float rt2 = 1.0f;
-        if (c->unit_kind == 0 && mean > 0.0f) rt2 = (range[base + u] * range[base + u]) / mean;
-        float w = G * rt2;
+        float R2 = 1.0f, rt2 = 1.0f;
+        if (c->unit_kind == 0) {
+            R2 = range[base + u] * range[base + u];
+            if (mean > 0.0f) rt2 = R2 / mean;
+        }
+        int us = (kind == 7) ? (int)(((long long)A * u + B0) % N) : u;
+        float w = weight_of(c, kind, ema_s[base + us], ema_r[base + us], R2, rt2);
         if (w > 0x1p60f) w = 0x1p60f;
         cw[u] = (w >= 0x1p-60f) ? w : -1.0f;  /* -1 flags the null weight 2^-200 (also NaN) */
     }
@@ -555,7 +601,11 @@ int orc_alloc(const orc_cfg* c, const float* ema_s, const float* ema_r, const fl
     long total = num / c->bbar_den;
     float* cw = (float*)malloc(sizeof(float) * N);
     for (int b = 0; b < c->B; b++) {
-        orc_weights(c, b, ema_s, ema_r, range, cw);
+        int rcw = orc_weights(c, b, ema_s, ema_r, range, cw);
+        if (rcw) {
+            free(cw);
+            return rcw;
+        }
         int rc = orc_alloc_from_weights(N, cw, c->bmin, c->bmax, total, c->bbar_num, c->bbar_den,
                                         widths + (size_t)b * N);
         if (rc) {

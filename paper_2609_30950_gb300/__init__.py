@@ -17,6 +17,9 @@ QSTATE_OK, QSTATE_EINVAL, QSTATE_EBUDGET, QSTATE_ECUDA, QSTATE_EDEVICE = range(5
 DECAY_ROW, DECAY_HEAD = 0, 1
 ERASE_DELTA, ERASE_NONE = 0, 1
 UNIT_ROW, UNIT_HEAD = 0, 1
+# allocation weights (Eq. 3 and the alternatives of Table 1; see include/qstate.h)
+(WEIGHT_OURS, WEIGHT_RANGE, WEIGHT_GAMMA_RAW, WEIGHT_NRANGE, WEIGHT_PERSIST, WEIGHT_WBFACTOR,
+ WEIGHT_NOERASE, WEIGHT_SHUFFLE, WEIGHT_UNIFORM) = range(9)
 
 
 class QstateError(RuntimeError):

@@ -68,6 +68,40 @@ __device__ int block_exclusive_scan(int v, int* red, int* total) {
 
 }  // namespace
 
+// Allocation weight c_u (Eq. 3 and the alternatives of Table 1), one IEEE rounding per
+// operation.  Rs / gmean: the batch element's ranges and group means of R^2 (row unit).
+__device__ float weight(const AllocParams& p, int u, size_t base, const float* Rs, const float* gmean, int gsz) {
+    const int kind = p.weight_kind;
+    float R2 = 1.0f, rt2 = 1.0f;   // R^2 and Rtilde^2 (1 for the head unit)
+    if (p.unit_row) {
+        const float R = Rs[u];
+        R2 = __fmul_rn(R, R);
+        const float m = gmean[u / gsz];
+        if (m > 0.0f) rt2 = __fdiv_rn(R2, m);
+    }
+    if (kind == QSTATE_WEIGHT_RANGE) return R2;
+    if (kind == QSTATE_WEIGHT_NRANGE) return rt2;
+    // statistics of the unit itself, or of unit pi(u) for the shuffled decay weights
+    const int us = kind == QSTATE_WEIGHT_SHUFFLE
+                       ? static_cast<int>((static_cast<long long>(p.shuf_a) * u + p.shuf_b) % p.units)
+                       : u;
+    const float ms = p.ema_s[base + us];
+    if (kind == QSTATE_WEIGHT_PERSIST) return __fmul_rn(__fdiv_rn(1.0f, ms), rt2);
+    if (kind == QSTATE_WEIGHT_WBFACTOR) {
+        float pw = 1.0f, bb = __fsub_rn(1.0f, ms);   // (1 - m_s)^C, low bit first
+        for (int e = p.C; e > 0; e >>= 1) {
+            if (e & 1) pw = __fmul_rn(pw, bb);
+            bb = __fmul_rn(bb, bb);
+        }
+        return __fmul_rn(__fdiv_rn(1.0f, __fsub_rn(1.0f, pw)), rt2);
+    }
+    float mr = kind == QSTATE_WEIGHT_NOERASE ? 0.0f : p.ema_r[base + us];
+    if (mr < 0.0f) mr = 0.0f;
+    const float G = __fdiv_rn(__fsub_rn(1.0f, ms), __fadd_rn(expm1_series(mr, p.e1), ms));
+    if (kind == QSTATE_WEIGHT_GAMMA_RAW) return __fmul_rn(G, R2);
+    return __fmul_rn(G, rt2);   // OURS, NOERASE, SHUFFLE
+}
+
 // Warp 0 only: the bin whose suffix count (bins >= it, highest first) first reaches `rank`
 // (1-based); returns it and sets *above to the count of the bins above it.  hist has 256 bins.
 __device__ int warp_select_bin(const int* hist, int rank, int* above) {
@@ -144,19 +178,7 @@ __global__ void __launch_bounds__(kThreads, 2) alloc_kernel(const AllocParams p)
     const long long M = p.total - static_cast<long long>(N) * p.bmin;
     for (int u = tid; u < N; u += kThreads) {
         float c = 1.0f;
-        if (!p.uniform) {
-            const float ms = p.ema_s[base + u];
-            float mr = p.ema_r[base + u];
-            if (mr < 0.0f) mr = 0.0f;
-            const float G = __fdiv_rn(__fsub_rn(1.0f, ms), __fadd_rn(expm1_series(mr, p.e1), ms));
-            float rt2 = 1.0f;
-            if (p.unit_row) {
-                const float m = gmean[u / gsz];
-                const float R = Rs[u];
-                if (m > 0.0f) rt2 = __fdiv_rn(__fmul_rn(R, R), m);
-            }
-            c = __fmul_rn(G, rt2);
-        }
+        if (!p.uniform) c = weight(p, u, base, Rs, gmean, gsz);
         if (c > 0x1p60f) c = 0x1p60f;
         const int k = (c >= 0x1p-60f) ? __float_as_int(c) : kNullKey;
         key[u] = k;

@@ -95,7 +95,8 @@ int validate(const qstate_cfg* c) {
     if (c->fit_every < 1) return fail(QSTATE_EINVAL, "fit_every must be >= 1");
     if (!(c->ema_span > 0.0f)) return fail(QSTATE_EINVAL, "ema_span must be > 0");
     if (c->gate_bits < 0 || c->gate_bits > 8) return fail(QSTATE_EINVAL, "gate_bits must be in [0, 8]");
-    if (c->weight_kind != QSTATE_WEIGHT_OURS) return fail(QSTATE_EINVAL, "unsupported weight_kind");
+    if (c->weight_kind < QSTATE_WEIGHT_OURS || c->weight_kind > QSTATE_WEIGHT_UNIFORM)
+        return fail(QSTATE_EINVAL, "unsupported weight_kind %d", c->weight_kind);
     return QSTATE_OK;
 }
 
@@ -178,6 +179,16 @@ void set_inputs(StepParams& p, const qstate_inputs* x) {
     p.beta = x->beta;
 }
 
+// The shuffled-decay bijection of N units: u -> (A u + N / 3) mod N with A the smallest
+// integer above 0.6180339887 N that is coprime to N.
+int gcd_int(int a, int b) { return b == 0 ? a : gcd_int(b, a % b); }
+void shuffle_params(int N, int* A, int* Bo) {
+    int a = static_cast<int>(0.6180339887 * N) + 1;
+    while (gcd_int(a, N) != 1) ++a;
+    *A = a % N;
+    *Bo = N / 3;
+}
+
 int run_alloc(const qstate_cfg* c, const float* ms, const float* mr, const float* range, int uniform,
               uint8_t* widths, uint32_t* head_off, int* status, cudaStream_t st) {
     AllocParams a;
@@ -192,7 +203,10 @@ int run_alloc(const qstate_cfg* c, const float* ms, const float* mr, const float
     a.bmin = c->bmin;
     a.bmax = c->bmax;
     a.total = units_of(c) * c->bbar_num / c->bbar_den;
-    a.uniform = uniform;
+    a.uniform = uniform || c->weight_kind == QSTATE_WEIGHT_UNIFORM;
+    a.weight_kind = c->weight_kind;
+    a.C = c->C;
+    shuffle_params(a.units, &a.shuf_a, &a.shuf_b);
     a.ema_s = ms;
     a.ema_r = mr;
     a.range = range;

@@ -63,6 +63,9 @@ struct AllocParams {
     int B, H, dk, dv, units, unit_row, group_heads, bmin, bmax;
     long long total;   // sum of widths per batch element
     int uniform;       // 1: ignore statistics, equal weights (initial widths)
+    int weight_kind;   // QSTATE_WEIGHT_*
+    int C;             // write-back period (write-back factor weight)
+    int shuf_a, shuf_b;   // shuffled-decay bijection u -> (shuf_a u + shuf_b) mod units
     const float* ema_s;
     const float* ema_r;
     const float* range;

@@ -70,6 +70,25 @@ def test_alloc_bit_exact(qs, orc, name):
         assert np.array_equal(host(head_off, np.uint32), oref), (name, trial)
 
 
+@pytest.mark.parametrize("kind", range(9))
+@pytest.mark.parametrize("name", ["kda_decode", "gdn_decode", "mamba2_decode"])
+def test_alloc_weight_kinds_bit_exact(qs, orc, name, kind):
+    """The allocation weights of Table 1 (weight_kind 1-8) give the oracle's widths bit for bit."""
+    w = synth.scaled(synth.WORKLOADS[name], B=3)
+    over = dict(weight_kind=kind, C=16 if kind == 5 else w.C)
+    cfgq, cfgo = qs.Config.from_workload(w, **over), orc.Cfg.from_workload(w, **over)
+    rng = np.random.default_rng(100 + kind)
+    ms, mr, R = _random_stats(cfgo, rng, null_rows=3)
+    st = qs.Stats(dev(ms, torch), dev(mr, torch), dev(R, torch))
+    widths = torch.zeros(cfgq.B * cfgq.units, dtype=torch.uint8, device="cuda")
+    head_off = torch.zeros(cfgq.B * cfgq.H, dtype=torch.int32, device="cuda")
+    qs.qstate_alloc_bits(cfgq, st, widths, head_off)
+    qs.qstate_check()
+    wref, oref = orc.alloc(cfgo, ms, mr, R)
+    assert np.array_equal(host(widths, np.uint8), wref)
+    assert np.array_equal(host(head_off, np.uint32), oref)
+
+
 @pytest.mark.parametrize("name", ["tiny_kda", "kda_decode", "gdn_decode", "mamba2_decode"])
 def test_init_bit_exact(qs, orc, name):
     w = synth.scaled(synth.WORKLOADS[name], B=2)
@@ -186,13 +205,13 @@ def test_fp32_recurrence_free_running(qs, orc, name):
 
 
 # --------------------------------------------------------------- quantised write-backs, lockstep
-def _lockstep(qs, orc, w, fit_every=1, log_decay=False, sample_b=None, max_wb=None):
+def _lockstep(qs, orc, w, fit_every=1, log_decay=False, sample_b=None, max_wb=None, weight_kind=0):
     """Run the oracle free; before every write-back copy its state into the GPU, run one
     qstate_step and compare the GPU's write-back with the oracle's.  With sample_b, the GPU
     runs the full batch and only those batch elements are injected and compared (the oracle
     runs a B=1 configuration per sampled element)."""
-    cfgq = qs.Config.from_workload(w, fit_every=fit_every)
-    cfgo_full = orc.Cfg.from_workload(w, fit_every=fit_every)
+    cfgq = qs.Config.from_workload(w, fit_every=fit_every, weight_kind=weight_kind)
+    cfgo_full = orc.Cfg.from_workload(w, fit_every=fit_every, weight_kind=weight_kind)
     inp = synth.host_inputs(w)
     s_code = s_lut = None
     if log_decay:
@@ -201,7 +220,8 @@ def _lockstep(qs, orc, w, fit_every=1, log_decay=False, sample_b=None, max_wb=No
     X, _ = _dev_inputs(w, inp, qs, s_code, s_lut)
     bs = list(range(w.B)) if sample_b is None else list(sample_b)
     one = sample_b is not None
-    cfgo = orc.Cfg.from_workload(synth.scaled(w, B=1), fit_every=fit_every) if one else cfgo_full
+    cfgo = (orc.Cfg.from_workload(synth.scaled(w, B=1), fit_every=fit_every, weight_kind=weight_kind)
+            if one else cfgo_full)
     sub = (lambda a, b: a[b:b + 1]) if one else (lambda a, b: a)
     orc_inp = {b: {k: sub(v, b) for k, v in inp.items()} for b in (bs if one else [0])}
     orc_code = {b: (sub(s_code, b) if s_code is not None else None) for b in (bs if one else [0])}
@@ -270,7 +290,8 @@ def _lockstep(qs, orc, w, fit_every=1, log_decay=False, sample_b=None, max_wb=No
             # of the same statistics must agree bit for bit (checked through qstate_alloc_bits)
             wn, on = orc.alloc(cfgo, S["ms"], S["mr"], S["R"])
             sts = qs.Stats(dev(S["ms"], torch), dev(S["mr"], torch), dev(S["R"], torch))
-            cq = qs.Config.from_workload(synth.scaled(w, B=cfgo.B), fit_every=fit_every)
+            cq = qs.Config.from_workload(synth.scaled(w, B=cfgo.B), fit_every=fit_every,
+                                         weight_kind=weight_kind)
             wt = torch.zeros(cfgo.B * units, dtype=torch.uint8, device="cuda")
             ot = torch.zeros(cfgo.B * w.H, dtype=torch.int32, device="cuda")
             qs.qstate_alloc_bits(cq, sts, wt, ot)
@@ -298,6 +319,13 @@ def test_quantised_lockstep(qs, orc, name):
 def test_quantised_lockstep_fit_every(qs, orc):
     w = small("kda_decode", B=2, H=4, T=10, gate_bits=0)
     _lockstep(qs, orc, w, fit_every=4)
+
+
+@pytest.mark.parametrize("kind", [5, 7])
+def test_quantised_lockstep_weight_kinds(qs, orc, kind):
+    """A scan with the write-back-factor or shuffled-decay weights (Table 1) stays in lockstep:
+    the allocation between write-backs uses the configured weight."""
+    _lockstep(qs, orc, SMALL["kda_decode"], log_decay=True, weight_kind=kind)
 
 
 def test_quantised_lockstep_ragged_chunks(qs, orc):
