@@ -305,7 +305,10 @@ def main():
     sha = kernel_sha()
     traffic = recorded_traffic(sha)
 
-    # end to end through the public API: pinned host inputs -> device, the step, o -> host
+    # end to end through the public API: pinned host inputs -> device, the step, o -> host.
+    # The rates go first (the log-decay levels are taken over all tokens of the step); q, k,
+    # v and beta then stream in chunk by chunk on a copy stream while the compute stream scans
+    # the previous chunk, and readouts stream back (qstate_scan_host).
     e2e = None
     if not args.no_e2e:
         names = ["q", "k", "v", "s", "beta"]
@@ -315,22 +318,28 @@ def main():
         host_o = torch.empty(o.shape, dtype=o.dtype, pin_memory=True)
         h2d = sum(t.numel() * t.element_size() for t in host_in.values())
         d2h = host_o.numel() * host_o.element_size()
+        comp, copy_stream = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+        comp.wait_stream(stream)
+        xh = q.Inputs(host_in["q"], host_in["k"], host_in["v"], None, None, None, host_in["beta"], w.T)
+        chunk = 64
 
         def e2e_step():
-            for n in names:
-                x[n].copy_(host_in[n], non_blocking=True)
-            step()
-            host_o.copy_(o, non_blocking=True)
+            with torch.cuda.stream(comp):
+                x["s"].copy_(host_in["s"], non_blocking=True)
+            q.qstate_quant_decay(cfg, x["s"], codes, lut, thr, comp)
+            q.qstate_init(cfg, A, Bst, comp)
+            q.qstate_scan_host(cfg, A, Bst, xh, X, 0, w.T, 0, host_o, o, st, chunk, comp,
+                               copy_stream)
 
         e2e_step()
         barrier()
         k2 = max(1, min(args.steps, 3))
         s0 = torch.cuda.Event(enable_timing=True)
         s1 = torch.cuda.Event(enable_timing=True)
-        s0.record(stream)
+        s0.record(comp)
         for _ in range(k2):
             e2e_step()
-        s1.record(stream)
+        s1.record(comp)
         barrier()
         e_ms = s0.elapsed_time(s1) / k2
         if world > 1:
@@ -338,8 +347,9 @@ def main():
             dist.all_reduce(t, op=dist.ReduceOp.MAX)
             e_ms = float(t.item())
         e2e = {"value": tokens_step * world / (e_ms / 1000.0), "unit": "tokens/s",
-               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e_ms}
-        q.qstate_check(stream)
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e_ms,
+               "staging": f"qstate_scan_host, {chunk}-token chunks on a copy stream"}
+        q.qstate_check(comp)
 
     launches_per_step = 4 + 2 + 2 * w.T   # decay (4), init (alloc + pack), T x (write-back + alloc)
     clocks = clk.summary()

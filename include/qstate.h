@@ -215,6 +215,23 @@ int qstate_scan(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong,
                 const qstate_inputs* x, int32_t t_begin, int32_t t_end, int32_t w_index0,
                 float* o, qstate_stats* stats, int32_t* final_in_pong, void* stream);
 
+/* qstate_scan fed from pinned host memory, for callers whose token inputs and readouts live
+ * on the host.  x_host and x_dev describe the same (B, T, H, .) tensors (same T) in host and
+ * device memory; every input present in x_host (q, k, v, beta, s or s_code) is copied, token
+ * chunk by token chunk, into x_dev's buffer with one 2D copy per tensor and chunk on
+ * copy_stream, while the compute stream runs the scan of the previous chunk; inputs absent
+ * from x_host (e.g. rate codes made on the device by qstate_quant_decay) must already be in
+ * x_dev.  Readouts of each chunk are copied from o_dev to o_host on copy_stream once the chunk
+ * is done.  chunk (tokens) is a multiple of C.  stream and copy_stream are distinct non-NULL
+ * streams; work on stream completes only after the last readout has reached o_host.  Host
+ * memory should be pinned (pageable memory works but the copies then serialise).  Results are
+ * those of qstate_scan(ping, pong, x_dev, ...) bit for bit. */
+int qstate_scan_host(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong,
+                     const qstate_inputs* x_host, const qstate_inputs* x_dev, int32_t t_begin,
+                     int32_t t_end, int32_t w_index0, float* o_host, float* o_dev,
+                     qstate_stats* stats, int32_t chunk, int32_t* final_in_pong, void* stream,
+                     void* copy_stream);
+
 /* Unquantised reference path: Eq. (1) on a dense FP32 state S (device, (B, H, dk, dv), in/out)
  * for tokens [t_begin, t_end), the state round-tripping through memory every C tokens. */
 int qstate_scan_fp32(const qstate_cfg* cfg, float* S, const qstate_inputs* x, int32_t t_begin,

@@ -56,7 +56,7 @@ class _Inputs(ct.Structure):
 EXPORTS = ["qstate_validate", "qstate_region_bytes", "qstate_units", "qstate_scale_groups",
            "qstate_bits_per_element", "qstate_init", "qstate_alloc_bits", "qstate_pack",
            "qstate_unpack", "qstate_quant_decay", "qstate_quant_decay_noalloc", "qstate_step",
-           "qstate_scan",
+           "qstate_scan", "qstate_scan_host",
            "qstate_scan_fp32", "qstate_check", "qstate_last_error"]
 
 _lib = None
@@ -98,6 +98,9 @@ def load(path: str | None = None, build_if_missing: bool = False):
     L.qstate_scan.argtypes = [PC, ct.POINTER(_Buf), ct.POINTER(_Buf), ct.POINTER(_Inputs),
                               ct.c_int32, ct.c_int32, ct.c_int32, P, ct.POINTER(_Stats),
                               ct.POINTER(ct.c_int32), P]
+    L.qstate_scan_host.argtypes = [PC, ct.POINTER(_Buf), ct.POINTER(_Buf), ct.POINTER(_Inputs),
+                                   ct.POINTER(_Inputs), ct.c_int32, ct.c_int32, ct.c_int32, P, P,
+                                   ct.POINTER(_Stats), ct.c_int32, ct.POINTER(ct.c_int32), P, P]
     L.qstate_scan_fp32.argtypes = [PC, P, ct.POINTER(_Inputs), ct.c_int32, ct.c_int32, P, P]
     L.qstate_check.argtypes = [P]
     L.qstate_last_error.restype = ct.c_char_p
@@ -304,6 +307,33 @@ def qstate_scan(cfg: Config, ping: State, pong: State, x: Inputs, t_begin: int, 
     _check(_lib_or_raise().qstate_scan(ct.byref(c), ct.byref(bi), ct.byref(bo), ct.byref(xi),
                                        t_begin, t_end, w_index0, _ptr(o), ct.byref(st),
                                        ct.byref(flag), _stream(stream)))
+    return bool(flag.value)
+
+
+def _hptr(t):
+    """Pointer of a host (CPU) tensor; pinned memory keeps the copies asynchronous."""
+    if t is None:
+        return None
+    if t.is_cuda or not t.is_contiguous():
+        raise ValueError("host tensor must be a contiguous CPU tensor")
+    return ct.c_void_p(t.data_ptr())
+
+
+def qstate_scan_host(cfg: Config, ping: State, pong: State, x_host: Inputs, x_dev: Inputs,
+                     t_begin: int, t_end: int, w_index0: int, o_host, o_dev, stats: Stats,
+                     chunk: int, stream, copy_stream) -> bool:
+    """qstate_scan with inputs staged from host tensors chunk by chunk (see include/qstate.h).
+    Returns True if the final state is in ``pong``."""
+    c, bi, bo, st = cfg.c(), ping.c(), pong.c(), stats.c()
+    xh = _Inputs(*(_hptr(getattr(x_host, n)) for n in ("q", "k", "v", "s", "s_code", "s_lut", "beta")),
+                 x_host.T or int(x_host.q.shape[1]))
+    xd = x_dev.c()
+    flag = ct.c_int32(0)
+    _check(_lib_or_raise().qstate_scan_host(ct.byref(c), ct.byref(bi), ct.byref(bo), ct.byref(xh),
+                                            ct.byref(xd), t_begin, t_end, w_index0, _hptr(o_host),
+                                            _ptr(o_dev), ct.byref(st), chunk, ct.byref(flag),
+                                            ct.c_void_p(stream.cuda_stream),
+                                            ct.c_void_p(copy_stream.cuda_stream)))
     return bool(flag.value)
 
 

@@ -433,6 +433,83 @@ int qstate_scan(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong, const
     return QSTATE_OK;
 }
 
+int qstate_scan_host(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong,
+                     const qstate_inputs* x_host, const qstate_inputs* x_dev, int32_t t_begin,
+                     int32_t t_end, int32_t w_index0, float* o_host, float* o_dev,
+                     qstate_stats* stats, int32_t chunk, int32_t* final_in_pong, void* stream,
+                     void* copy_stream) {
+    int rc = validate(cfg);
+    if (rc) return rc;
+    if ((rc = check_inputs(cfg, x_dev, t_begin, t_end, o_dev))) return rc;
+    if (!x_host || !o_host || x_host->T != x_dev->T)
+        return fail(QSTATE_EINVAL, "host inputs / readouts missing or of another length");
+    if (!stream || !copy_stream || stream == copy_stream)
+        return fail(QSTATE_EINVAL, "need two distinct non-default streams");
+    if (chunk < 1 || chunk % cfg->C != 0) return fail(QSTATE_EINVAL, "chunk must be a multiple of C");
+    // every input given on the host side must have a device buffer to land in
+    const bool bad = (x_host->q && !x_dev->q) || (x_host->k && !x_dev->k) || (x_host->v && !x_dev->v) ||
+                     (x_host->beta && !x_dev->beta) || (x_host->s && !x_dev->s) ||
+                     (x_host->s_code && !x_dev->s_code);
+    if (bad) return fail(QSTATE_EINVAL, "a host input has no device buffer");
+    cudaStream_t cs = static_cast<cudaStream_t>(stream), ts = static_cast<cudaStream_t>(copy_stream);
+    const int B = cfg->B, T = x_dev->T, H = cfg->H;
+    const size_t f4 = sizeof(float);
+    const size_t nchan = cfg->decay_kind == QSTATE_DECAY_ROW ? static_cast<size_t>(H) * cfg->dk : H;
+    struct Item { void* d; const void* h; size_t per; };
+    const Item in[6] = {{(void*)x_dev->q, x_host->q, H * cfg->dk * f4}, {(void*)x_dev->k, x_host->k, H * cfg->dk * f4},
+                        {(void*)x_dev->v, x_host->v, H * cfg->dv * f4}, {(void*)x_dev->beta, x_host->beta, H * f4},
+                        {(void*)x_dev->s, x_host->s, nchan * f4}, {(void*)x_dev->s_code, x_host->s_code, nchan}};
+    // tokens [t0, t1) of a (B, T, per) token-major tensor: one 2D copy, rows = batch elements
+    auto copy_tokens = [&](void* dst, const void* src, size_t per, int t0, int t1, cudaMemcpyKind kind) {
+        const size_t pitch = static_cast<size_t>(T) * per, off = static_cast<size_t>(t0) * per;
+        return cudaMemcpy2DAsync(static_cast<char*>(dst) + off, pitch, static_cast<const char*>(src) + off,
+                                 pitch, static_cast<size_t>(t1 - t0) * per, B, kind, ts);
+    };
+    qstate_buf* src = ping;
+    qstate_buf* dst = pong;
+    int in_pong = 0, w = w_index0;
+    cudaError_t e = cudaSuccess;
+    cudaEvent_t ev_in = nullptr, ev_out = nullptr;
+    for (int c0 = t_begin; c0 < t_end && e == cudaSuccess && rc == QSTATE_OK; c0 += chunk) {
+        const int c1 = c0 + chunk < t_end ? c0 + chunk : t_end;
+        for (const Item& it : in)
+            if (it.h && e == cudaSuccess) e = copy_tokens(it.d, it.h, it.per, c0, c1, cudaMemcpyHostToDevice);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev_in, cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaEventRecord(ev_in, ts);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, ev_in, 0);
+        if (ev_in) cudaEventDestroy(ev_in);
+        ev_in = nullptr;
+        if (e != cudaSuccess) break;
+        int flip = 0;
+        rc = qstate_scan(cfg, src, dst, x_dev, c0, c1, w, o_dev, stats, &flip, stream);
+        if (rc) break;
+        w += (c1 - c0 + cfg->C - 1) / cfg->C;
+        if (flip) {
+            qstate_buf* tmp = src;
+            src = dst;
+            dst = tmp;
+            in_pong ^= 1;
+        }
+        e = cudaEventCreateWithFlags(&ev_out, cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaEventRecord(ev_out, cs);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(ts, ev_out, 0);
+        if (ev_out) cudaEventDestroy(ev_out);
+        ev_out = nullptr;
+        if (e == cudaSuccess) e = copy_tokens(o_host, o_dev, H * cfg->dv * f4, c0, c1, cudaMemcpyDeviceToHost);
+    }
+    // the compute stream completes only after the last readout copy
+    if (e == cudaSuccess && rc == QSTATE_OK) {
+        e = cudaEventCreateWithFlags(&ev_out, cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaEventRecord(ev_out, ts);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, ev_out, 0);
+        if (ev_out) cudaEventDestroy(ev_out);
+    }
+    if (rc) return rc;
+    if (e != cudaSuccess) return cuda_fail(e, "host staging");
+    if (final_in_pong) *final_in_pong = in_pong;
+    return QSTATE_OK;
+}
+
 int qstate_scan_fp32(const qstate_cfg* cfg, float* S, const qstate_inputs* x, int32_t t_begin,
                      int32_t t_end, float* o, void* stream) {
     int rc = validate(cfg);

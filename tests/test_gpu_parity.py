@@ -403,3 +403,68 @@ def test_scan_equals_repeated_steps(qs, orc):
     assert np.array_equal(outs[0][0], outs[1][0])
     for f in ("payload", "scales", "widths", "head_off", "fidx"):
         assert np.array_equal(getattr(outs[0][1], f), getattr(outs[1][1], f))
+
+
+# ------------------------------------------------------------------ host-staged scan
+@pytest.mark.parametrize("name,chunk", [("kda_decode", 3), ("gdn_decode", 4), ("kda_prefill", 8)])
+def test_scan_host_equals_scan(qs, orc, name, chunk):
+    """qstate_scan_host (inputs copied from pinned host memory chunk by chunk on a second
+    stream) gives qstate_scan's readouts and final state bit for bit."""
+    w = SMALL[name]
+    if name == "kda_prefill":
+        w = synth.scaled(w, T=2 * w.C + 5)
+        chunk = w.C
+    cfgq = qs.Config.from_workload(w)
+    inp = synth.host_inputs(w)
+    s_code = s_lut = None
+    if w.gate_bits:
+        nchan = w.H * w.dk if w.per_row_decay else w.H
+        s_code, s_lut, _ = orc.quant_decay(inp["s"], nchan, w.gate_bits)
+    X, _ = _dev_inputs(w, inp, qs, s_code, s_lut)
+    # reference: device inputs
+    A, Bs, st = qs.new_state(cfgq), qs.new_state(cfgq), qs.new_stats(cfgq)
+    qs.qstate_init(cfgq, A, Bs)
+    o_ref = torch.zeros((w.B, w.T, w.H, w.dv), dtype=torch.float32, device="cuda")
+    pong_ref = qs.qstate_scan(cfgq, A, Bs, X, 0, w.T, 0, o_ref, st)
+    qs.qstate_check()
+    # host-staged: device buffers start as garbage and are filled chunk by chunk
+    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
+    xh = qs.Inputs(pin(inp["q"]), pin(inp["k"]), pin(inp["v"]),
+                   None if s_code is not None else pin(inp["s"]), None, None,
+                   pin(inp["beta"]) if w.erase else None, w.T)
+    xd = qs.Inputs(torch.full_like(X.q, 7.0), torch.full_like(X.k, 7.0), torch.full_like(X.v, 7.0),
+                   None if X.s is None else torch.full_like(X.s, 7.0), X.s_code, X.s_lut,
+                   None if X.beta is None else torch.full_like(X.beta, 7.0), w.T)
+    A2, B2, st2 = qs.new_state(cfgq), qs.new_state(cfgq), qs.new_stats(cfgq)
+    qs.qstate_init(cfgq, A2, B2)
+    o_dev = torch.zeros_like(o_ref)
+    o_host = torch.zeros(o_ref.shape, dtype=torch.float32).pin_memory()
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    s1.wait_stream(torch.cuda.current_stream())
+    pong = qs.qstate_scan_host(cfgq, A2, B2, xh, xd, 0, w.T, 0, o_host, o_dev, st2, chunk, s1, s2)
+    s1.synchronize()
+    qs.qstate_check()
+    assert pong == pong_ref
+    assert np.array_equal(o_host.numpy().view(np.uint32), host(o_ref, np.float32).view(np.uint32))
+    fin, fin2 = (Bs, B2) if pong else (A, A2)
+    for f in ("payload", "scales", "widths", "head_off", "fidx"):
+        assert torch.equal(getattr(fin, f), getattr(fin2, f)), f
+    for f in ("ema_s", "ema_r", "range"):
+        assert torch.equal(getattr(st, f), getattr(st2, f)), f
+
+
+def test_scan_host_argument_errors(qs):
+    w = SMALL["kda_decode"]
+    cfgq = qs.Config.from_workload(w, gate_bits=0)
+    inp = synth.host_inputs(w)
+    X, _ = _dev_inputs(w, inp, qs)
+    A, Bs, st = qs.new_state(cfgq), qs.new_state(cfgq), qs.new_stats(cfgq)
+    xh = qs.Inputs(*(torch.from_numpy(np.ascontiguousarray(inp[n])) for n in ("q", "k", "v", "s")),
+                   None, None, torch.from_numpy(np.ascontiguousarray(inp["beta"])), w.T)
+    o = torch.zeros((w.B, w.T, w.H, w.dv), dtype=torch.float32, device="cuda")
+    oh = torch.zeros(o.shape, dtype=torch.float32)
+    s1 = torch.cuda.Stream()
+    with pytest.raises(qs.QstateError):        # one stream for both roles
+        qs.qstate_scan_host(cfgq, A, Bs, xh, X, 0, w.T, 0, oh, o, st, 2, s1, s1)
+    with pytest.raises(qs.QstateError):        # chunk not a multiple of C (C = 1: chunk 0)
+        qs.qstate_scan_host(cfgq, A, Bs, xh, X, 0, w.T, 0, oh, o, st, 0, s1, torch.cuda.Stream())
