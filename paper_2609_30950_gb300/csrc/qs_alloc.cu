@@ -150,7 +150,7 @@ __global__ void __launch_bounds__(kThreads, 2) alloc_kernel(const AllocParams p)
     float* Rs = reinterpret_cast<float*>(key + N);                   // row unit: ranges
     float* gmean = Rs + (p.unit_row ? N : 0);
     int* hist = reinterpret_cast<int*>(gmean + ((ngroups + 3) & ~3));
-    int* redi = hist + 256;
+    int* redi = hist + 1024;                                           // hist: 256 bins, then H head sizes
     int* sel = redi + 72;                                              // H*, rank, low prefix
     uint8_t* wv = reinterpret_cast<uint8_t*>(sel + 4);
     const int tid = threadIdx.x;
@@ -182,10 +182,19 @@ __global__ void __launch_bounds__(kThreads, 2) alloc_kernel(const AllocParams p)
         if (c > 0x1p60f) c = 0x1p60f;
         const int k = (c >= 0x1p-60f) ? __float_as_int(c) : kNullKey;
         key[u] = k;
-        if (J > 0) {
-            const int E = k >> 24;   // in [-37, 127]
-            atomicAdd(&hist[E - J + kHistOff], 1);
-            atomicAdd(&hist[E + kHistOff], -1);
+    }
+    // lanes with equal high parts add together (one atomic per distinct value and warp)
+    if (J > 0) {
+        for (int u0w = tid - (tid & 31); u0w < N; u0w += kThreads) {
+            const int u = u0w + (tid & 31);
+            const bool in = u < N;
+            const int E = in ? (key[u] >> 24) : 0x7fffffff;   // in [-37, 127]
+            const unsigned peers = __match_any_sync(kFull, E);
+            if (in && (tid & 31) == __ffs(peers) - 1) {
+                const int cnt = __popc(peers);
+                atomicAdd(&hist[E - J + kHistOff], cnt);
+                atomicAdd(&hist[E + kHistOff], -cnt);
+            }
         }
     }
     __syncthreads();
@@ -285,18 +294,23 @@ __global__ void __launch_bounds__(kThreads, 2) alloc_kernel(const AllocParams p)
     }
     __syncthreads();
 
-    // 5. head offsets: exclusive prefix sum of the heads' payload bytes
-    int hb = 0;
-    for (int h = tid; h < p.H; h += kThreads) {   // H <= 1024 (validated)
-        if (p.unit_row) {
-            for (int i = 0; i < p.dk; ++i) hb += wv[h * p.dk + i];
-            hb *= p.dv / 8;
-        } else {
-            hb = wv[h] * p.dk * p.dv / 8;
+    // 5. head offsets: exclusive prefix sum of the heads' payload bytes (row unit: one warp
+    //    per head sums its widths)
+    int* hbytes = hist;   // free again
+    if (p.unit_row) {
+        for (int h = tid >> 5; h < p.H; h += kThreads / 32) {
+            int sum = 0;
+            for (int i = tid & 31; i < p.dk; i += 32) sum += wv[h * p.dk + i];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(kFull, sum, o);
+            if ((tid & 31) == 0) hbytes[h] = sum * (p.dv / 8);
         }
+    } else {
+        for (int h = tid; h < p.H; h += kThreads) hbytes[h] = wv[h] * p.dk * p.dv / 8;
     }
+    __syncthreads();
     int total_bytes = 0;
-    const int off = block_exclusive_scan(tid < p.H ? hb : 0, redi, &total_bytes);
+    const int off = block_exclusive_scan(tid < p.H ? hbytes[tid] : 0, redi, &total_bytes);
     if (tid < p.H) p.head_off[static_cast<size_t>(blockIdx.x) * p.H + tid] = static_cast<uint32_t>(off);
     if (tid == 0 && M > 0 && (need < 1 || need > tie_total)) raise_status(p.status, QS_DEV_LAYOUT);
 }
@@ -304,7 +318,7 @@ __global__ void __launch_bounds__(kThreads, 2) alloc_kernel(const AllocParams p)
 cudaError_t launch_alloc(const AllocParams& p, cudaStream_t stream) {
     const int ngroups = p.unit_row ? p.units / (p.group_heads * p.dk) : 0;
     const size_t smem = static_cast<size_t>(p.units) * 4 + (p.unit_row ? p.units * 4 : 0) +
-                        ((ngroups + 3) & ~3) * 4 + 256 * 4 + 72 * 4 + 4 * 4 + p.units + 16;
+                        ((ngroups + 3) & ~3) * 4 + 1024 * 4 + 72 * 4 + 4 * 4 + p.units + 16;
     cudaError_t e = cudaFuncSetAttribute(alloc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
