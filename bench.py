@@ -200,6 +200,28 @@ def run_reference(args, w):
     print(json.dumps(line))
 
 
+def slowest_ms(ms, world, device):
+    """Max over ranks of a per-rank time (ms); the job is as fast as its slowest rank."""
+    if world <= 1:
+        return float(ms)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(tokens_per_rank, world, ms):
+    """Whole-job tokens/s: every rank runs its own batch of independent sequences (weak scaling,
+    no exchange on the data path), so the job processes world x tokens_per_rank per step."""
+    return tokens_per_rank * world / (ms / 1000.0)
+
+
+def rank_seed_offset(rank):
+    """Each rank draws its own batch of sequences (a shard of the job's batch)."""
+    return rank
+
+
 def config_of(w, args):
     return {"workload": w.name, "B": w.B, "H": w.H, "dk": w.dk, "dv": w.dv, "T": w.T, "C": w.C,
             "bbar": w.bbar, "widths": [w.bmin, w.bmax], "gate_bits": w.gate_bits,
@@ -240,7 +262,7 @@ def main():
     q.load(build_if_missing=True)
 
     cfg = q.Config.from_workload(w, fit_every=args.fit_every)
-    x = synth.device_inputs(w, device=dev, seed_offset=rank)
+    x = synth.device_inputs(w, device=dev, seed_offset=rank_seed_offset(rank))
     nchan = w.H * w.dk
     L = 1 << w.gate_bits
     codes = torch.empty(x["s"].shape, dtype=torch.uint8, device=dev)
@@ -287,14 +309,10 @@ def main():
         barrier()
         wall = time.perf_counter() - t0
     q.qstate_check(stream)
-    ms_total = start.elapsed_time(end)
-    if world > 1:
-        t = torch.tensor([ms_total], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_total = float(t.item())
+    ms_total = slowest_ms(start.elapsed_time(end), world, dev)
     ms_step = ms_total / args.steps
     tokens_step = w.B * w.T
-    value = tokens_step * world / (ms_step / 1000.0)
+    value = job_throughput(tokens_step, world, ms_step)
     scan_ms = statistics.median(e1.elapsed_time(e2) for _, e1, e2 in ev)
     decay_ms = statistics.median(e0.elapsed_time(e1) for e0, e1, _ in ev)
     per_wb_ms = scan_ms / w.T        # write-back kernel + allocation kernel per token
@@ -341,12 +359,8 @@ def main():
             e2e_step()
         s1.record(comp)
         barrier()
-        e_ms = s0.elapsed_time(s1) / k2
-        if world > 1:
-            t = torch.tensor([e_ms], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e_ms = float(t.item())
-        e2e = {"value": tokens_step * world / (e_ms / 1000.0), "unit": "tokens/s",
+        e_ms = slowest_ms(s0.elapsed_time(s1) / k2, world, dev)
+        e2e = {"value": job_throughput(tokens_step, world, e_ms), "unit": "tokens/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e_ms,
                "staging": f"qstate_scan_host, {chunk}-token chunks on a copy stream"}
         q.qstate_check(comp)

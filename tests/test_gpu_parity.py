@@ -335,12 +335,18 @@ def test_quantised_lockstep_ragged_chunks(qs, orc):
 
 @pytest.mark.parametrize("name,T,sample", [("kda_decode", 3, (0, 131, 255)),
                                            ("gdn_decode", 3, (0, 63)),
-                                           ("mamba2_decode", 2, (5, 127))])
+                                           ("mamba2_decode", 2, (5, 127)),
+                                           ("kda_prefill", 70, (0, 15))])
 def test_full_size_sampled_lockstep(qs, orc, name, T, sample):
     """Full batch and heads of the benchmark workloads, in the launch configuration the
     benchmark times; sampled batch elements are compared write-back by write-back."""
     w = synth.scaled(synth.WORKLOADS[name], T=T)
     _lockstep(qs, orc, w, log_decay=(w.gate_bits > 0), sample_b=sample)
+
+
+def test_tiny_kda_full_lockstep(qs, orc):
+    """The tiny recurrence at its full length (T = 256 per-token write-backs)."""
+    _lockstep(qs, orc, synth.WORKLOADS["tiny_kda"])
 
 
 # ---------------------------------------------------------------------------------- edge cases
