@@ -48,6 +48,7 @@ extern "C" {
 #define QSTATE_DECAY_HEAD 1  /* one rate per head (Gated DeltaNet, Mamba-2)                   */
 #define QSTATE_ERASE_DELTA 0 /* a = beta k, w = beta 1 (Eq. 1, KDA / Gated DeltaNet)          */
 #define QSTATE_ERASE_NONE 1  /* a = 0, w = 1 (Eq. 1, Mamba-2)                                  */
+#define QSTATE_ERASE_GENERAL 2 /* a and w given per token (Eq. 1 in general)                  */
 #define QSTATE_UNIT_ROW 0    /* width + FP16 scale per row (Sec. 3, "Allocation units")       */
 #define QSTATE_UNIT_HEAD 1   /* width per head, FP16 scale per 32 key rows x value column     */
 /* Allocation weights c_i (Eq. 3 and the alternatives of Table 1).  With the EMAs of
@@ -119,9 +120,14 @@ typedef struct qstate_stats {
 } qstate_stats;
 
 /* Token inputs (device).  q, k: (B, T, H, dk); v: (B, T, H, dv); s: (B, T, H, dk) for per-row
- * decay or (B, T, H) for per-head decay, all rates > 0; beta: (B, T, H), ignored without
- * erasure.  With log-quantised rates pass s = NULL, s_code (uint8, same shape as s) and
- * s_lut (channels x 2^gate_bits levels, channels = H*dk or H) from qstate_quant_decay. */
+ * decay or (B, T, H) for per-head decay, all rates > 0; beta: (B, T, H), used by
+ * QSTATE_ERASE_DELTA only.  With log-quantised rates pass s = NULL, s_code (uint8, same shape
+ * as s) and s_lut (channels x 2^gate_bits levels, channels = H*dk or H) from
+ * qstate_quant_decay.  a: (B, T, H, dk) and w: (B, T, H, dv), used by QSTATE_ERASE_GENERAL
+ * only: S = (I - k a^T) D S + k (w o v)^T.  Its erasure statistic (the EMA behind Eq. 3's r_i)
+ * is 2 a_i k_i - a_i^2 |k|^2, the fraction of row i's error energy one token removes, which
+ * is beta (2 - beta) k_i^2 for a = beta k and a unit key (row unit); the head unit averages
+ * it over the rows. */
 typedef struct qstate_inputs {
     const float* q;
     const float* k;
@@ -131,6 +137,8 @@ typedef struct qstate_inputs {
     const float* s_lut;
     const float* beta;
     int32_t T;
+    const float* a;
+    const float* w;
 } qstate_inputs;
 
 /* ---- sizes and accounting (host only) ---------------------------------------------------- */

@@ -52,7 +52,7 @@ class Cfg:
     dk: int
     dv: int
     decay_kind: int = 0      # 0 per row, 1 per head
-    erase_kind: int = 0      # 0 delta rule, 1 none
+    erase_kind: int = 0      # 0 delta rule, 1 none, 2 general (a, w given per token)
     unit_kind: int = 0       # 0 row unit, 1 head unit
     group_heads: int = 1
     bbar_num: int = 4
@@ -83,7 +83,8 @@ class Cfg:
     @classmethod
     def from_workload(cls, w, **over) -> "Cfg":
         kw = dict(B=w.B, H=w.H, dk=w.dk, dv=w.dv, decay_kind=0 if w.per_row_decay else 1,
-                  erase_kind=0 if w.erase else 1, unit_kind=0 if w.unit == "row" else 1,
+                  erase_kind=(2 if getattr(w, "general", False) else 0 if w.erase else 1),
+                  unit_kind=0 if w.unit == "row" else 1,
                   group_heads=w.group_heads, bbar_num=w.bbar, bbar_den=1, bmin=w.bmin,
                   bmax=w.bmax, C=w.C, gate_bits=w.gate_bits)
         kw.update(over)
@@ -121,7 +122,7 @@ def lib():
         L.orc_alloc.argtypes = [ct.POINTER(OrcCfg), P, P, P, P, P]
         L.orc_init_widths.argtypes = [ct.POINTER(OrcCfg), P, P]
         L.orc_quant_decay.argtypes = [ct.c_long, ct.c_int, P, ct.c_int, P, P, P]
-        L.orc_step.argtypes = ([ct.POINTER(OrcCfg)] + [P] * 10 + [ct.c_int] * 4 + [P] * 12)
+        L.orc_step.argtypes = ([ct.POINTER(OrcCfg)] + [P] * 10 + [ct.c_int] * 4 + [P] * 14)
     return _lib
 
 
@@ -169,6 +170,9 @@ def expand_inputs(cfg: Cfg, inp: dict, b: int, h: int):
         beta = inp["beta"][b, :, h].astype(np.float32)
         a = (beta[:, None] * k).astype(np.float32)
         w = np.repeat(beta[:, None], cfg.dv, axis=1).astype(np.float32)
+    elif cfg.erase_kind == 2:
+        a = inp["a"][b, :, h].astype(np.float32)
+        w = inp["w"][b, :, h].astype(np.float32)
     else:
         a = np.zeros_like(k)
         w = np.ones((T, cfg.dv), np.float32)
@@ -362,13 +366,15 @@ def step(cfg: Cfg, src: Buf, dst: Buf, inp: dict, t_begin, t_end, w_index, o, em
     q, k, v = (_c(inp[n], np.float32) for n in ("q", "k", "v"))
     s = None if s_code is not None else _c(inp["s"], np.float32)
     beta = _c(inp["beta"], np.float32)
+    a_in = _c(inp["a"], np.float32) if "a" in inp else None
+    w_in = _c(inp["w"], np.float32) if "w" in inp else None
     sc = None if s_code is None else _c(s_code, np.uint8)
     sl = None if s_lut is None else _c(s_lut, np.float32)
     rc = lib().orc_step(ct.byref(c), _p(src.payload), _p(src.scales), _p(src.widths),
                         _p(src.head_off), _p(src.fidx), _p(dst.payload), _p(dst.scales),
                         _p(dst.widths), _p(dst.head_off), _p(dst.fidx), T, t_begin, t_end,
                         w_index, _p(q), _p(k), _p(v), _p(s), _p(sc), _p(sl), _p(beta), _p(o),
-                        _p(ema_s), _p(ema_r), _p(rng), _p(x))
+                        _p(ema_s), _p(ema_r), _p(rng), _p(x), _p(a_in), _p(w_in))
     _check(rc, "step")
     return x
 

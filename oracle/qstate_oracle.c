@@ -701,7 +701,11 @@ int orc_quant_decay(long count, int nchan, const float* s, int g, uint8_t* codes
  * (B, T, H) for per-head rates; with s_code/s_lut the rate is s_lut[ch * 2^g + code].
  * EMA per token (span 64): alpha = 2 / (span + 1), m <- m + alpha (x - m), the first token
  * of the sequence (t = 0) initialising m = x; x_s = 1 - e^{-2 s}, x_r = beta (2 - beta) k_i^2
- * (row unit) or beta (2 - beta) |k|^2 / dk (head unit), 0 without erasure.
+ * (row unit) or beta (2 - beta) |k|^2 / dk (head unit), 0 without erasure.  With general
+ * erasure (erase_kind 2) a_tok (B, T, H, dk) and w_tok (B, T, H, dv) give a and w per token
+ * and x_r = 2 a_i k_i - a_i^2 |k|^2 (row unit) or its mean over the rows (head unit): the
+ * fraction of row i's error energy that (I - k a^T) removes, beta (2 - beta) k_i^2 for
+ * a = beta k and |k| = 1.
  * The range factor is refitted when fit_every <= 1 or (w_index + h) % fit_every == 0, else
  * the factor stored at the previous write-back (fidx_in) is reused.
  * x_dump (optional) receives the FP32 state before quantisation (B, H, dk, dv).
@@ -711,10 +715,12 @@ int orc_step(const orc_cfg* c, const uint8_t* pay_in, const uint16_t* sc_in, con
              const uint8_t* w_out, const uint32_t* off_out, uint8_t* fidx_out, int T, int t_begin,
              int t_end, int w_index, const float* q, const float* k, const float* v,
              const float* s, const uint8_t* s_code, const float* s_lut, const float* beta,
-             float* o, float* ema_s, float* ema_r, float* range, float* x_dump) {
+             float* o, float* ema_s, float* ema_r, float* range, float* x_dump,
+             const float* a_tok, const float* w_tok) {
     int H = c->H, dk = c->dk, dv = c->dv, L = 1 << c->gate_bits;
     long rb = orc_region_bytes(c);
     if (rb < 0 || !layout_ok(c, w_in, off_in) || !layout_ok(c, w_out, off_out)) return ORC_EINVAL;
+    if (c->erase_kind == 2 && (!a_tok || !w_tok)) return ORC_EINVAL;
     float alpha = 2.0f / (c->ema_span + 1.0f);
     float* X = (float*)malloc(sizeof(float) * (size_t)dk * dv);
     float* d = (float*)malloc(sizeof(float) * dk);
@@ -727,6 +733,12 @@ int orc_step(const orc_cfg* c, const uint8_t* pay_in, const uint16_t* sc_in, con
                 size_t tok = ((size_t)b * T + t) * H + h;
                 const float *kt = k + tok * dk, *qt = q + tok * dk, *vt = v + tok * dv;
                 float bt = (c->erase_kind == 0) ? beta[tok] : 1.0f;
+                /* general erasure (erase_kind 2): a, w given; its statistic per row is
+                 * 2 a_i k_i - a_i^2 |k|^2 (|k|^2 summed in index order) */
+                const float *at = (c->erase_kind == 2) ? a_tok + tok * dk : 0;
+                const float *wt = (c->erase_kind == 2) ? w_tok + tok * dv : 0;
+                float ksq = 0.0f;
+                for (int i = 0; i < dk; i++) ksq = ksq + kt[i] * kt[i];
                 float ssum = 0.0f;
                 for (int i = 0; i < dk; i++) {
                     int ch = (c->decay_kind == 0) ? h * dk + i : h;
@@ -738,6 +750,7 @@ int orc_step(const orc_cfg* c, const uint8_t* pay_in, const uint16_t* sc_in, con
                         size_t u = ((size_t)b * H + h) * dk + i;
                         float xs = -expm1f(-2.0f * si_rate);
                         float xr = (c->erase_kind == 0) ? (bt * (2.0f - bt)) * (kt[i] * kt[i]) : 0.0f;
+                        if (c->erase_kind == 2) xr = 2.0f * (at[i] * kt[i]) - (at[i] * at[i]) * ksq;
                         if (t == 0) {
                             ema_s[u] = xs;
                             ema_r[u] = xr;
@@ -752,6 +765,14 @@ int orc_step(const orc_cfg* c, const uint8_t* pay_in, const uint16_t* sc_in, con
                     size_t u = (size_t)b * H + h;
                     float xs = -expm1f(-2.0f * (s_code ? s_lut[(size_t)h * L + s_code[tok]] : s[tok]));
                     float xr = (c->erase_kind == 0) ? (bt * (2.0f - bt)) * (ssum / (float)dk) : 0.0f;
+                    if (c->erase_kind == 2) {   /* mean over rows of 2 a_i k_i - a_i^2 |k|^2 */
+                        float ak = 0.0f, aa = 0.0f;
+                        for (int i = 0; i < dk; i++) {
+                            ak = ak + at[i] * kt[i];
+                            aa = aa + at[i] * at[i];
+                        }
+                        xr = (2.0f * ak - aa * ksq) / (float)dk;
+                    }
                     if (t == 0) {
                         ema_s[u] = xs;
                         ema_r[u] = xr;
@@ -773,6 +794,16 @@ int orc_step(const orc_cfg* c, const uint8_t* pay_in, const uint16_t* sc_in, con
                         for (int j = 0; j < dv; j++)
                             X[(size_t)i * dv + j] =
                                 (X[(size_t)i * dv + j] - kt[i] * p[j]) + kt[i] * (bt * vt[j]);
+                } else if (c->erase_kind == 2) {   /* Eq. (1) with the given a and w */
+                    for (int j = 0; j < dv; j++) {
+                        float acc = 0.0f;
+                        for (int i = 0; i < dk; i++) acc = acc + at[i] * X[(size_t)i * dv + j];
+                        p[j] = acc;
+                    }
+                    for (int i = 0; i < dk; i++)
+                        for (int j = 0; j < dv; j++)
+                            X[(size_t)i * dv + j] =
+                                (X[(size_t)i * dv + j] - kt[i] * p[j]) + kt[i] * (wt[j] * vt[j]);
                 } else {
                     for (int i = 0; i < dk; i++)
                         for (int j = 0; j < dv; j++)

@@ -15,7 +15,7 @@ from . import build as _build
 
 QSTATE_OK, QSTATE_EINVAL, QSTATE_EBUDGET, QSTATE_ECUDA, QSTATE_EDEVICE = range(5)
 DECAY_ROW, DECAY_HEAD = 0, 1
-ERASE_DELTA, ERASE_NONE = 0, 1
+ERASE_DELTA, ERASE_NONE, ERASE_GENERAL = 0, 1, 2
 UNIT_ROW, UNIT_HEAD = 0, 1
 # allocation weights (Eq. 3 and the alternatives of Table 1; see include/qstate.h)
 (WEIGHT_OURS, WEIGHT_RANGE, WEIGHT_GAMMA_RAW, WEIGHT_NRANGE, WEIGHT_PERSIST, WEIGHT_WBFACTOR,
@@ -50,7 +50,7 @@ class _Stats(ct.Structure):
 class _Inputs(ct.Structure):
     _fields_ = [("q", ct.c_void_p), ("k", ct.c_void_p), ("v", ct.c_void_p), ("s", ct.c_void_p),
                 ("s_code", ct.c_void_p), ("s_lut", ct.c_void_p), ("beta", ct.c_void_p),
-                ("T", ct.c_int32)]
+                ("T", ct.c_int32), ("a", ct.c_void_p), ("w", ct.c_void_p)]
 
 
 EXPORTS = ["qstate_validate", "qstate_region_bytes", "qstate_units", "qstate_scale_groups",
@@ -165,7 +165,8 @@ class Config:
     def from_workload(cls, w, **over) -> "Config":
         kw = dict(B=w.B, H=w.H, dk=w.dk, dv=w.dv,
                   decay_kind=DECAY_ROW if w.per_row_decay else DECAY_HEAD,
-                  erase_kind=ERASE_DELTA if w.erase else ERASE_NONE,
+                  erase_kind=(ERASE_GENERAL if getattr(w, "general", False)
+                            else ERASE_DELTA if w.erase else ERASE_NONE),
                   unit_kind=UNIT_ROW if w.unit == "row" else UNIT_HEAD,
                   group_heads=w.group_heads, bbar_num=w.bbar, bbar_den=1, bmin=w.bmin,
                   bmax=w.bmax, C=w.C, gate_bits=w.gate_bits)
@@ -248,11 +249,13 @@ class Inputs:
     s_lut: object = None
     beta: object = None
     T: int = field(default=0)
+    a: object = None
+    w: object = None
 
     def c(self) -> _Inputs:
         T = self.T or int(self.q.shape[1])
         return _Inputs(_ptr(self.q), _ptr(self.k), _ptr(self.v), _ptr(self.s), _ptr(self.s_code),
-                       _ptr(self.s_lut), _ptr(self.beta), T)
+                       _ptr(self.s_lut), _ptr(self.beta), T, _ptr(self.a), _ptr(self.w))
 
 
 def qstate_init(cfg: Config, a: State, b: State, stream=None) -> None:
@@ -326,7 +329,7 @@ def qstate_scan_host(cfg: Config, ping: State, pong: State, x_host: Inputs, x_de
     Returns True if the final state is in ``pong``."""
     c, bi, bo, st = cfg.c(), ping.c(), pong.c(), stats.c()
     xh = _Inputs(*(_hptr(getattr(x_host, n)) for n in ("q", "k", "v", "s", "s_code", "s_lut", "beta")),
-                 x_host.T or int(x_host.q.shape[1]))
+                 x_host.T or int(x_host.q.shape[1]), _hptr(x_host.a), _hptr(x_host.w))
     xd = x_dev.c()
     flag = ct.c_int32(0)
     _check(_lib_or_raise().qstate_scan_host(ct.byref(c), ct.byref(bi), ct.byref(bo), ct.byref(xh),

@@ -72,7 +72,8 @@ int validate(const qstate_cfg* c) {
     if (!shape_ok) return fail(QSTATE_EINVAL, "unsupported (dk, dv) = (%d, %d)", c->dk, c->dv);
     if (c->decay_kind != QSTATE_DECAY_ROW && c->decay_kind != QSTATE_DECAY_HEAD)
         return fail(QSTATE_EINVAL, "bad decay_kind");
-    if (c->erase_kind != QSTATE_ERASE_DELTA && c->erase_kind != QSTATE_ERASE_NONE)
+    if (c->erase_kind != QSTATE_ERASE_DELTA && c->erase_kind != QSTATE_ERASE_NONE &&
+        c->erase_kind != QSTATE_ERASE_GENERAL)
         return fail(QSTATE_EINVAL, "bad erase_kind");
     if (c->unit_kind != QSTATE_UNIT_ROW && c->unit_kind != QSTATE_UNIT_HEAD)
         return fail(QSTATE_EINVAL, "bad unit_kind");
@@ -146,6 +147,7 @@ StepParams base_params(const qstate_cfg* c, int* status) {
     p.B = c->B;
     p.H = c->H;
     p.erase = c->erase_kind == QSTATE_ERASE_DELTA ? 1 : 0;
+    p.general = c->erase_kind == QSTATE_ERASE_GENERAL ? 1 : 0;
     p.decay_row = c->decay_kind == QSTATE_DECAY_ROW ? 1 : 0;
     p.fit_every = c->fit_every;
     p.L = c->gate_bits > 0 ? (1 << c->gate_bits) : 0;
@@ -159,6 +161,8 @@ StepParams base_params(const qstate_cfg* c, int* status) {
 int check_inputs(const qstate_cfg* c, const qstate_inputs* x, int t_begin, int t_end, const float* o) {
     if (!x || !x->q || !x->k || !x->v || !o) return fail(QSTATE_EINVAL, "null input or output pointer");
     if (c->erase_kind == QSTATE_ERASE_DELTA && !x->beta) return fail(QSTATE_EINVAL, "beta is NULL");
+    if (c->erase_kind == QSTATE_ERASE_GENERAL && (!x->a || !x->w))
+        return fail(QSTATE_EINVAL, "general erasure needs a and w");
     if (x->s_code) {
         if (c->gate_bits < 1 || !x->s_lut) return fail(QSTATE_EINVAL, "s_code needs gate_bits >= 1 and s_lut");
     } else if (!x->s) {
@@ -177,6 +181,8 @@ void set_inputs(StepParams& p, const qstate_inputs* x) {
     p.s_code = x->s_code;
     p.s_lut = x->s_lut;
     p.beta = x->beta;
+    p.a_in = x->a;
+    p.w_in = x->w;
 }
 
 // The shuffled-decay bijection of N units: u -> (A u + N / 3) mod N with A the smallest
@@ -449,16 +455,18 @@ int qstate_scan_host(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong,
     // every input given on the host side must have a device buffer to land in
     const bool bad = (x_host->q && !x_dev->q) || (x_host->k && !x_dev->k) || (x_host->v && !x_dev->v) ||
                      (x_host->beta && !x_dev->beta) || (x_host->s && !x_dev->s) ||
-                     (x_host->s_code && !x_dev->s_code);
+                     (x_host->s_code && !x_dev->s_code) || (x_host->a && !x_dev->a) ||
+                     (x_host->w && !x_dev->w);
     if (bad) return fail(QSTATE_EINVAL, "a host input has no device buffer");
     cudaStream_t cs = static_cast<cudaStream_t>(stream), ts = static_cast<cudaStream_t>(copy_stream);
     const int B = cfg->B, T = x_dev->T, H = cfg->H;
     const size_t f4 = sizeof(float);
     const size_t nchan = cfg->decay_kind == QSTATE_DECAY_ROW ? static_cast<size_t>(H) * cfg->dk : H;
     struct Item { void* d; const void* h; size_t per; };
-    const Item in[6] = {{(void*)x_dev->q, x_host->q, H * cfg->dk * f4}, {(void*)x_dev->k, x_host->k, H * cfg->dk * f4},
+    const Item in[8] = {{(void*)x_dev->q, x_host->q, H * cfg->dk * f4}, {(void*)x_dev->k, x_host->k, H * cfg->dk * f4},
                         {(void*)x_dev->v, x_host->v, H * cfg->dv * f4}, {(void*)x_dev->beta, x_host->beta, H * f4},
-                        {(void*)x_dev->s, x_host->s, nchan * f4}, {(void*)x_dev->s_code, x_host->s_code, nchan}};
+                        {(void*)x_dev->s, x_host->s, nchan * f4}, {(void*)x_dev->s_code, x_host->s_code, nchan},
+                        {(void*)x_dev->a, x_host->a, H * cfg->dk * f4}, {(void*)x_dev->w, x_host->w, H * cfg->dv * f4}};
     // tokens [t0, t1) of a (B, T, per) token-major tensor: one 2D copy, rows = batch elements
     auto copy_tokens = [&](void* dst, const void* src, size_t per, int t0, int t1, cudaMemcpyKind kind) {
         const size_t pitch = static_cast<size_t>(T) * per, off = static_cast<size_t>(t0) * per;

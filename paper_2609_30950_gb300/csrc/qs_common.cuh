@@ -54,6 +54,17 @@ __device__ __forceinline__ float code_magic(float x, float inv, float lo, float 
     return fminf(fmaxf(t, lo), hi);
 }
 
+// Erasure statistic of a row under general erasure (Eq. (1) with a given a):
+// 2 a_i k_i - a_i^2 |k|^2, the fraction of the row's error energy that (I - k a^T) removes;
+// |k|^2 summed in index order over the DK entries of kvec, one rounding per operation.
+template <int DK>
+__device__ __forceinline__ float general_erasure(float ai, float ki, const float* kvec) {
+    float ksq = 0.0f;
+#pragma unroll 8
+    for (int r = 0; r < DK; ++r) ksq = __fadd_rn(ksq, __fmul_rn(kvec[r], kvec[r]));
+    return __fsub_rn(__fmul_rn(2.0f, __fmul_rn(ai, ki)), __fmul_rn(__fmul_rn(ai, ai), ksq));
+}
+
 // ---- warp reductions ----------------------------------------------------------------------
 __device__ __forceinline__ float warp_absmax(float v) {
     unsigned m = __reduce_max_sync(kFull, __float_as_uint(fabsf(v)));

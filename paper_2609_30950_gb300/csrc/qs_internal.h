@@ -21,7 +21,8 @@ constexpr int kNFit = 16;
 struct StepParams {
     int B, H, T;
     int t_begin, t_end, w_index;
-    int erase;        // 1: delta rule (a = beta k, w = beta 1); 0: a = 0, w = 1
+    int erase;        // 1: delta rule (a = beta k, w = beta 1); 0: a = 0, w = 1 (or general)
+    int general;      // 1: a and w given per token (a_in, w_in)
     int decay_row;    // 1: per-row rates; 0: per-head rates
     int fit_every;
     int L;            // 2^gate_bits (0 when rates are FP32)
@@ -51,6 +52,8 @@ struct StepParams {
     const uint8_t* s_code;
     const float* s_lut;
     const float* beta;
+    const float* a_in;
+    const float* w_in;
     float* o;
     // statistics (may be null when there are no tokens)
     float* ema_s;

@@ -34,6 +34,7 @@ struct alignas(16) StepSmem {
     float cand[HEAD ? 1 : DK][kNFit][2];  // row unit: (Delta_k, 1/Delta_k) of the refit rows
     float k[DK], q[DK], d[DK];
     float v[DV], u[DV];
+    float ga[DK], gw[DV];                 // general erasure: this token's a and w
     float red[2][NW][DV];                 // p and r partials per warp
     float scale_in[NSG];                  // source steps / means (float)
     float ms[DK], mr[DK];                 // EMA statistics (head unit uses [0])
@@ -43,7 +44,7 @@ struct alignas(16) StepSmem {
     float colmax[HEAD ? NW * DV : 1];     // head unit: per-warp column maxima / sums
     float fitf[kNFit];                    // f_k = (5 + k) / 20
     float inv_n[17];                      // 1 / (2^(w-1) - 1), w = 2..16
-    float wsum[2][NW];                    // per-warp partial k.q and |k|^2
+    float wsum[4][NW];                    // per-warp partial k.q, |k|^2, a.k, |a|^2
     int off_in[DK + 1], off_out[DK + 1];  // row byte offsets inside the head (+ total)
     uint16_t out_scale[NSG];
     uint8_t out_fidx[NSG];
@@ -256,7 +257,11 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
                                 : __ldg(p.s + tok * DK + i);
             if (!(rate > 0.0f) || !(rate < INFINITY)) raise_status(p.status, QS_DEV_RATE);
             sm.d[i] = expf(-rate);
-            if (stats && !HEAD) {   // Sec. 3 statistics per row
+            const float ai = p.general ? __ldg(p.a_in + tok * DK + i) : __fmul_rn(beta, kk);
+            sm.ga[i] = ai;
+            // Sec. 3 statistics per row (general erasure: after the barrier, as the erasure
+            // term needs all of k)
+            if (stats && !HEAD && !p.general) {
                 const float xs = -expm1f(-2.0f * rate);
                 const float xr = p.erase ? __fmul_rn(__fmul_rn(beta, __fsub_rn(2.0f, beta)), __fmul_rn(kk, kk)) : 0.0f;
                 if (t == 0) {
@@ -269,13 +274,37 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
             }
             const float kq = warp_sum(kk * qq);
             const float k2 = warp_sum(kk * kk);
+            const float ak = warp_sum(ai * kk);
+            const float aa = warp_sum(ai * ai);
             if (lane == 0) {
                 sm.wsum[0][warp] = kq;
                 sm.wsum[1][warp] = k2;
+                sm.wsum[2][warp] = ak;
+                sm.wsum[3][warp] = aa;
             }
         }
-        if (tid < DV) sm.v[tid] = __ldg(p.v + tok * DV + tid);
+        if (tid < DV) {
+            sm.v[tid] = __ldg(p.v + tok * DV + tid);
+            if (p.general) sm.gw[tid] = __ldg(p.w_in + tok * DV + tid);
+        }
         __syncthreads();
+        if (stats && !HEAD && p.general && tid < DK) {   // Sec. 3 statistics per row
+            const int i = tid;
+            float rate = rate_h;
+            if (p.decay_row)
+                rate = p.s_code ? __ldg(p.s_lut + (static_cast<size_t>(h) * DK + i) * p.L +
+                                        min(static_cast<int>(p.s_code[tok * DK + i]), p.L - 1))
+                                : __ldg(p.s + tok * DK + i);
+            const float xs = -expm1f(-2.0f * rate);
+            const float xr = general_erasure<DK>(sm.ga[i], sm.k[i], sm.k);
+            if (t == 0) {
+                sm.ms[i] = xs;
+                sm.mr[i] = xr;
+            } else {
+                sm.ms[i] = __fadd_rn(sm.ms[i], __fmul_rn(p.alpha, __fsub_rn(xs, sm.ms[i])));
+                sm.mr[i] = __fadd_rn(sm.mr[i], __fmul_rn(p.alpha, __fsub_rn(xr, sm.mr[i])));
+            }
+        }
 
         // decay and per-lane partial reductions over the warp's rows
         float pp[CPL], rr[CPL];
@@ -285,7 +314,7 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
         for (int r = 0; r < RPW; ++r) {
             const int i = warp * RPW + r;
             const float d = sm.d[i];
-            const float a = __fmul_rn(beta, sm.k[i]);   // erase vector a = beta k
+            const float a = sm.ga[i];   // erase vector: beta k (delta rule) or the given a
             const float qi = sm.q[i];
 #pragma unroll
             for (int c = 0; c < CPL; ++c) {
@@ -312,7 +341,8 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
             for (int w = 0; w < DK / 32; ++w) kq += sm.wsum[0][w];
             const float vj = sm.v[j];
             // S = S' - k (a^T S') + k (w o v)^T:  u = beta v - p (delta rule), u = v (no erase)
-            const float u = p.erase ? __fsub_rn(__fmul_rn(beta, vj), P) : vj;
+            const float wj = p.general ? sm.gw[j] : beta;
+            const float u = (p.erase || p.general) ? __fsub_rn(__fmul_rn(wj, vj), P) : vj;
             sm.u[j] = u;
             p.o[tok * DV + j] = fmaf(u, kq, Rr);   // o = S^T q = S'^T q + u (k . q)
         }
@@ -321,9 +351,18 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
 #pragma unroll
             for (int w = 0; w < DK / 32; ++w) k2 += sm.wsum[1][w];
             const float xs = -expm1f(-2.0f * rate_h);
-            const float xr = p.erase ? __fmul_rn(__fmul_rn(beta, __fsub_rn(2.0f, beta)),
-                                                 __fdiv_rn(k2, static_cast<float>(DK)))
-                                     : 0.0f;
+            float xr = p.erase ? __fmul_rn(__fmul_rn(beta, __fsub_rn(2.0f, beta)),
+                                           __fdiv_rn(k2, static_cast<float>(DK)))
+                               : 0.0f;
+            if (p.general) {   // mean over the rows of 2 a_i k_i - a_i^2 |k|^2
+                float ak = 0.0f, aa = 0.0f;
+#pragma unroll
+                for (int w = 0; w < DK / 32; ++w) {
+                    ak += sm.wsum[2][w];
+                    aa += sm.wsum[3][w];
+                }
+                xr = __fdiv_rn(__fsub_rn(__fmul_rn(2.0f, ak), __fmul_rn(aa, k2)), static_cast<float>(DK));
+            }
             if (t == 0) {
                 sm.ms[0] = xs;
                 sm.mr[0] = xr;

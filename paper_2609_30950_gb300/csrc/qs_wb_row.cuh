@@ -53,6 +53,7 @@ struct alignas(16) WbStage {
     float ms[DK], mr[DK], k[DK], q[DK], s[DK];
     float v[DV];
     float lut[DK * 4];                           // the head's decay levels (when 2^g <= 4)
+    float ga[DK], gw[DV];                        // general erasure: the first token's a and w
     float beta, rate_h, pad0, pad1;
     int in_off, in_end, out_off, ok;              // payload window of this head
     int nxt_in_off, nxt_in_end, nxt_out_off, pad2;   // offsets of the following head
@@ -79,6 +80,7 @@ struct alignas(16) WbSmem {
     float4 deq[DK];                       // (-A, S, B, 0): x = (2^23 + u - A) S + B
     float4 wc[17];                        // per width: (n, 1/n, 2^23*1.5 - n, 2^23*1.5 + n)
     float tk[DK], tq[DK], tv[DV];         // inputs of tokens after the first (C > 1)
+    float tw[DV];                         // general erasure: w of tokens after the first
     float a[DK], d[DK];                   // erase vector beta k, decay of the current token
     float u[DV];
     float rowR[DK];
@@ -302,6 +304,13 @@ __device__ __noinline__ void wb_issue_meta(WbStage<DK, DV>& S, int g, int gnext,
     } else if ((c -= C32) < C8) {
         if (p.decay_row && p.s_code) cp_async16(S.scode + 16 * c, p.s_code + tok * DK + 16 * c);
     }
+    // general erasure: the first token's a (DK floats) and w (DV floats)
+    if (p.general) {
+        for (int i = tid; i < DK / 4 + DV / 4; i += blockDim.x) {
+            if (i < DK / 4) cp_async16(S.ga + 4 * i, p.a_in + tok * DK + 4 * i);
+            else cp_async16(S.gw + 4 * (i - DK / 4), p.w_in + tok * DV + 4 * (i - DK / 4));
+        }
+    }
     // the head's decay levels (DK x L floats, 16-byte chunks) when L <= 4
     if (p.decay_row && p.s_code && p.L <= 4) {
         const int nch = DK * p.L / 4;
@@ -462,9 +471,11 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
             }
             if (!(rate > 0.0f) || !(rate < INFINITY)) raise_status(p.status, QS_DEV_RATE);
             const float d = expf(-rate);
+            const float ai = p.general ? S.ga[i] : __fmul_rn(beta0, kk);
             if (stats) {
                 const float xs = -expm1f(-2.0f * rate);
-                const float xr = p.erase ? __fmul_rn(__fmul_rn(beta0, __fsub_rn(2.0f, beta0)), __fmul_rn(kk, kk)) : 0.0f;
+                float xr = p.erase ? __fmul_rn(__fmul_rn(beta0, __fsub_rn(2.0f, beta0)), __fmul_rn(kk, kk)) : 0.0f;
+                if (p.general) xr = general_erasure<DK>(ai, kk, S.k);
                 if (p.t_begin == 0) {
                     S.ms[i] = xs;
                     S.mr[i] = xr;
@@ -478,7 +489,7 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
             const float A = 8388608.0f + (w >= 2 ? sm.wc[w].x : 0.0f);
             sm.deq[i] = make_float4(-A, (w >= 2 ? D : (w == 1 ? -2.0f * D : 0.0f)) * d,
                                     (w == 1 ? D : 0.0f) * d, 0.0f);
-            sm.a[i] = __fmul_rn(beta0, kk);
+            sm.a[i] = ai;
             // k . q: one partial per warp of rows
             const float kq = warp_sum(kk * S.q[i]);
             if (lane == 0) sm.wsum[(tid - 64) >> 5] = kq;
@@ -569,18 +580,31 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                                         : __ldg(p.s + tok * DK + i);
                     if (!(rate > 0.0f) || !(rate < INFINITY)) raise_status(p.status, QS_DEV_RATE);
                     sm.d[i] = expf(-rate);
-                    sm.a[i] = __fmul_rn(beta, kk);
+                    sm.a[i] = p.general ? __ldg(p.a_in + tok * DK + i) : __fmul_rn(beta, kk);
                     if (stats) {
                         const float xs = -expm1f(-2.0f * rate);
-                        const float xr = p.erase ? __fmul_rn(__fmul_rn(beta, __fsub_rn(2.0f, beta)), __fmul_rn(kk, kk)) : 0.0f;
-                        S.ms[i] = __fadd_rn(S.ms[i], __fmul_rn(p.alpha, __fsub_rn(xs, S.ms[i])));
-                        S.mr[i] = __fadd_rn(S.mr[i], __fmul_rn(p.alpha, __fsub_rn(xr, S.mr[i])));
+                        if (p.general) {
+                            sm.rowR[i] = xs;   // the erasure term needs all of k: after the barrier
+                        } else {
+                            const float xr = p.erase ? __fmul_rn(__fmul_rn(beta, __fsub_rn(2.0f, beta)), __fmul_rn(kk, kk)) : 0.0f;
+                            S.ms[i] = __fadd_rn(S.ms[i], __fmul_rn(p.alpha, __fsub_rn(xs, S.ms[i])));
+                            S.mr[i] = __fadd_rn(S.mr[i], __fmul_rn(p.alpha, __fsub_rn(xr, S.mr[i])));
+                        }
                     }
                     const float s2 = warp_sum(kk * qq);
                     if (lane == 0) sm.wsum[warp] = s2;
                 }
-                if (tid < DV) sm.tv[tid] = __ldg(p.v + tok * DV + tid);
+                if (tid < DV) {
+                    sm.tv[tid] = __ldg(p.v + tok * DV + tid);
+                    if (p.general) sm.tw[tid] = __ldg(p.w_in + tok * DV + tid);
+                }
                 __syncthreads();
+                if (p.general && stats && tid < DK) {
+                    const float xs = sm.rowR[tid];
+                    const float xr = general_erasure<DK>(sm.a[tid], sm.tk[tid], sm.tk);
+                    S.ms[tid] = __fadd_rn(S.ms[tid], __fmul_rn(p.alpha, __fsub_rn(xs, S.ms[tid])));
+                    S.mr[tid] = __fadd_rn(S.mr[tid], __fmul_rn(p.alpha, __fsub_rn(xr, S.mr[tid])));
+                }
                 kv = sm.tk;
                 qv = sm.tq;
                 vv = sm.tv;
@@ -628,7 +652,9 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
 #pragma unroll
                 for (int w = 0; w < DK / 32; ++w) kq += sm.wsum[w];
                 const float vj = vv[jv];
-                const float uu = p.erase ? __fsub_rn(__fmul_rn(beta, vj), P) : vj;
+                // u = w o v - p (w = beta 1 for the delta rule; a = 0, w = 1 without erasure)
+                const float wj = p.general ? (t > p.t_begin ? sm.tw[jv] : S.gw[jv]) : beta;
+                const float uu = (p.erase || p.general) ? __fsub_rn(__fmul_rn(wj, vj), P) : vj;
                 sm.u[jv] = uu;
                 p.o[tok * DV + jv] = fmaf(uu, kq, Rr);
             }

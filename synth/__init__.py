@@ -24,6 +24,8 @@ import numpy as np
 KDA = "kda"        # per-row decay, delta-rule erase (a = beta k, w = beta 1)
 GDN = "gdn"        # per-head decay, delta-rule erase
 MAMBA2 = "mamba2"  # per-head decay, no erase (a = 0, w = 1)
+KDA_GEN = "kda_general"   # per-row decay, a and w drawn per token (Eq. (1) in general)
+GDN_GEN = "gdn_general"   # per-head decay, a and w drawn per token
 
 
 @dataclass(frozen=True)
@@ -50,11 +52,16 @@ class Workload:
 
     @property
     def per_row_decay(self) -> bool:
-        return self.family == KDA
+        return self.family in (KDA, KDA_GEN)
 
     @property
     def erase(self) -> bool:
         return self.family != MAMBA2
+
+    @property
+    def general(self) -> bool:
+        """a and w given per token instead of beta k and beta 1."""
+        return self.family in (KDA_GEN, GDN_GEN)
 
 
 # The five layer workloads: a tiny KDA recurrence, KDA decode, Gated DeltaNet decode,
@@ -71,6 +78,15 @@ WORKLOADS = {
                               kq_std=float(1.0 / np.sqrt(128.0)), seed=3000),
     "kda_prefill": Workload("kda_prefill", KDA, B=16, H=32, dk=128, dv=128, T=8192, C=64, bbar=3,
                             bmin=1, bmax=8, unit="row", seed=4000),
+}
+
+# Beyond the paper's layers: Eq. (1) with a and w given per token (a perturbed delta-rule
+# erase vector, per-channel write gates).
+EXTENSION_WORKLOADS = {
+    "kda_general": Workload("kda_general", KDA_GEN, B=32, H=8, dk=128, dv=128, T=256, C=1, bbar=4,
+                            bmin=1, bmax=8, unit="row", seed=5000),
+    "gdn_general": Workload("gdn_general", GDN_GEN, B=16, H=16, dk=128, dv=128, T=256, C=1, bbar=4,
+                            bmin=2, bmax=16, unit="head", s_loc=-3.0, seed=6000),
 }
 
 
@@ -90,7 +106,7 @@ def _sigmoid(z: np.ndarray) -> np.ndarray:
 
 
 # stream ids inside one workload seed
-_Q, _K, _V, _S, _BETA = 1, 2, 3, 4, 5
+_Q, _K, _V, _S, _BETA, _A, _W = 1, 2, 3, 4, 5, 6, 7
 
 
 def _rng(seed: int, stream: int, b: int, t: int) -> np.random.Generator:
@@ -121,6 +137,9 @@ def host_inputs(w: Workload, b_range=None, t_range=None) -> dict:
     v = np.empty((nb, nt, H, dv), np.float32)
     s = np.empty((nb, nt, H, dk) if w.per_row_decay else (nb, nt, H), np.float32)
     beta = np.empty((nb, nt, H), np.float32)
+    if w.general:
+        a = np.empty((nb, nt, H, dk), np.float32)
+        wg = np.empty((nb, nt, H, dv), np.float32)
     for bi in range(nb):
         for ti in range(nt):
             b, t = b0 + bi, t0 + ti
@@ -130,7 +149,14 @@ def host_inputs(w: Workload, b_range=None, t_range=None) -> dict:
             shape = (H, dk) if w.per_row_decay else (H,)
             s[bi, ti] = _softplus(w.s_loc + _rng(w.seed, _S, b, t).standard_normal(shape))
             beta[bi, ti] = _sigmoid(_rng(w.seed, _BETA, b, t).standard_normal((H,)))
-    return dict(q=q, k=k, v=v, s=s, beta=beta)
+            if w.general:
+                g = _rng(w.seed, _A, b, t).standard_normal((H, dk)) / np.sqrt(dk)
+                a[bi, ti] = beta[bi, ti][:, None] * (k[bi, ti] + 0.1 * g)
+                wg[bi, ti] = _sigmoid(_rng(w.seed, _W, b, t).standard_normal((H, dv)))
+    out = dict(q=q, k=k, v=v, s=s, beta=beta)
+    if w.general:
+        out.update(a=a, w=wg)
+    return out
 
 
 def device_inputs(w: Workload, device="cuda", T=None, seed_offset=0):
@@ -154,7 +180,12 @@ def device_inputs(w: Workload, device="cuda", T=None, seed_offset=0):
     shape = (B, T, H, dk) if w.per_row_decay else (B, T, H)
     s = torch.nn.functional.softplus(torch.randn(shape, **f32).add_(w.s_loc))
     beta = torch.sigmoid(torch.randn((B, T, H), **f32))
-    return dict(q=q, k=k, v=v, s=s, beta=beta)
+    out = dict(q=q, k=k, v=v, s=s, beta=beta)
+    if w.general:
+        g = torch.randn((B, T, H, dk), **f32).div_(dk ** 0.5)
+        out["a"] = beta[..., None] * (k + 0.1 * g)
+        out["w"] = torch.sigmoid(torch.randn((B, T, H, dv), **f32))
+    return out
 
 
 def random_state(w: Workload, seed: int, scale: float = 1.0) -> np.ndarray:

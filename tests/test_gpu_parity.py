@@ -30,10 +30,11 @@ SMALL = {
 
 def _dev_inputs(w, inp, q, s_code=None, s_lut=None):
     d = {k: dev(v, torch) for k, v in inp.items()}
+    a, wg = d.get("a"), d.get("w")
     if s_code is not None:
         return q.Inputs(d["q"], d["k"], d["v"], None, dev(s_code, torch), dev(s_lut, torch),
-                        d["beta"], w.T), d
-    return q.Inputs(d["q"], d["k"], d["v"], d["s"], None, None, d["beta"], w.T), d
+                        d["beta"], w.T, a, wg), d
+    return q.Inputs(d["q"], d["k"], d["v"], d["s"], None, None, d["beta"], w.T, a, wg), d
 
 
 def _random_stats(cfg, rng, zero_group=False, null_rows=0):
@@ -319,6 +320,33 @@ def test_quantised_lockstep(qs, orc, name):
 def test_quantised_lockstep_fit_every(qs, orc):
     w = small("kda_decode", B=2, H=4, T=10, gate_bits=0)
     _lockstep(qs, orc, w, fit_every=4)
+
+
+@pytest.mark.parametrize("name", ["kda_general", "gdn_general"])
+def test_general_erasure_lockstep(qs, orc, name):
+    """Eq. (1) with a and w given per token (row unit and head unit) stays in lockstep."""
+    w = synth.scaled(synth.EXTENSION_WORKLOADS[name], B=3, H=4, T=10)
+    _lockstep(qs, orc, w)
+
+
+@pytest.mark.parametrize("name", ["kda_general", "gdn_general"])
+def test_general_erasure_fp32_free_running(qs, orc, name):
+    """The unquantised FP32 recurrence with general a and w against the oracle's recurrence."""
+    w = synth.scaled(synth.EXTENSION_WORKLOADS[name], B=2, H=3, T=64)
+    cfgq, cfgo = qs.Config.from_workload(w), orc.Cfg.from_workload(w)
+    inp = synth.host_inputs(w)
+    X, _ = _dev_inputs(w, inp, qs)
+    S = torch.zeros((w.B, w.H, w.dk, w.dv), dtype=torch.float32, device="cuda")
+    o = torch.zeros((w.B, w.T, w.H, w.dv), dtype=torch.float32, device="cuda")
+    qs.qstate_scan_fp32(cfgq, S, X, 0, w.T, o)
+    qs.qstate_check()
+    og = host(o, np.float32)
+    worst = 0.0
+    for b in range(w.B):
+        for h in range(w.H):
+            o32, _ = orc.recur(np.zeros((w.dk, w.dv)), *orc.expand_inputs(cfgo, inp, b, h), dtype=np.float32)
+            worst = max(worst, rel_err_vectors(og[b, :, h], o32))
+    assert worst <= REL_O_FP32
 
 
 @pytest.mark.parametrize("kind", [5, 7])

@@ -236,3 +236,64 @@ def test_chunked_ragged_tail_matches_token_loop_without_quantisation_error(orc):
     ref, _ = orc.recur(np.zeros((w.dk, w.dv), np.float32), *orc.expand_inputs(cfg, inp, 0, 0))
     assert np.array_equal(o[0, :16, 0], ref[:16])
     assert np.all(np.isfinite(o))
+
+
+def _general_from_delta(inp):
+    """General-erasure inputs that reproduce the delta rule: a = fl(beta k), w = beta 1."""
+    g = dict(inp)
+    g["a"] = (inp["beta"][..., None] * inp["k"]).astype(np.float32)
+    g["w"] = np.repeat(inp["beta"][..., None], inp["v"].shape[-1], axis=-1).astype(np.float32)
+    return g
+
+
+def test_general_erasure_reproduces_delta_rule(orc):
+    """With a = beta k and w = beta 1 the general form of Eq. (1) is the delta rule: the same
+    readouts and packed state bit for bit; its erasure statistic 2 a_i k_i - a_i^2 |k|^2 is
+    beta (2 - beta) k_i^2 up to rounding for unit keys."""
+    w = _small("kda_decode", B=2, H=3, T=6)
+    inp = synth.host_inputs(w)
+    gin = _general_from_delta(inp)
+    res = {}
+    for kind, data in ((0, inp), (2, gin)):
+        cfg = orc.Cfg.from_workload(w, erase_kind=kind, gate_bits=0)
+        src, dst = orc.init_state(cfg)
+        o = np.zeros((w.B, w.T, w.H, w.dv), np.float32)
+        ms, mr, R = (np.zeros(cfg.B * cfg.units, np.float32) for _ in range(3))
+        for t in range(w.T):
+            orc.step(cfg, src, dst, data, t, t + 1, t, o, ms, mr, R)
+            src.widths[:], src.head_off[:] = orc.alloc(cfg, ms, mr, R) if t == 0 else (dst.widths, dst.head_off)
+            src, dst = dst, src
+        res[kind] = (o.copy(), src.payload.copy(), ms.copy(), mr.copy())
+    assert np.array_equal(res[0][0], res[2][0])
+    assert np.array_equal(res[0][1], res[2][1])
+    assert np.array_equal(res[0][2], res[2][2])
+    assert np.allclose(res[0][3], res[2][3], rtol=2e-6, atol=1e-9)
+
+
+def test_general_erasure_step_matches_recurrence(orc):
+    """The quantised scan with general a and w at 16 bits follows the unquantised general
+    recurrence (a second, independent implementation of Eq. (1) in the oracle)."""
+    w = synth.scaled(synth.EXTENSION_WORKLOADS["kda_general"], B=1, H=1, dk=64, dv=64, T=40,
+                     bbar=16, bmin=16, bmax=16)
+    cfg = orc.Cfg.from_workload(w)
+    assert cfg.erase_kind == 2
+    inp = synth.host_inputs(w)
+    o, *_ = orc.scan(cfg, inp)
+    ref, _ = orc.recur(np.zeros((w.dk, w.dv)), *orc.expand_inputs(cfg, inp, 0, 0), dtype=np.float64)
+    rel = np.linalg.norm(o[0, :, 0] - ref, axis=1) / np.linalg.norm(ref, axis=1)
+    assert rel.max() < 5e-3
+    # and it is not the delta rule: the perturbed a and the write gates change the readouts
+    dref, _ = orc.recur(np.zeros((w.dk, w.dv)),
+                        *orc.expand_inputs(orc.Cfg.from_workload(w, erase_kind=0), inp, 0, 0),
+                        dtype=np.float64)
+    assert np.linalg.norm(ref - dref) > 0.1 * np.linalg.norm(ref)
+
+
+def test_general_erasure_needs_a_and_w(orc):
+    w = _small("kda_decode", B=1, H=1, T=2)
+    cfg = orc.Cfg.from_workload(w, erase_kind=2, gate_bits=0)
+    src, dst = orc.init_state(cfg)
+    o = np.zeros((1, w.T, 1, w.dv), np.float32)
+    z = lambda: np.zeros(cfg.B * cfg.units, np.float32)
+    with pytest.raises(ValueError):
+        orc.step(cfg, src, dst, synth.host_inputs(w), 0, 1, 0, o, z(), z(), z())
