@@ -225,7 +225,8 @@ def rank_seed_offset(rank):
 def config_of(w, args):
     return {"workload": w.name, "B": w.B, "H": w.H, "dk": w.dk, "dv": w.dv, "T": w.T, "C": w.C,
             "bbar": w.bbar, "widths": [w.bmin, w.bmax], "gate_bits": w.gate_bits,
-            "fit_every": args.fit_every, "global_batch": w.B * args.gpus, "seq_len": w.T,
+            "fit_every": args.fit_every, "alloc_mode": getattr(args, "alloc_mode", 0),
+            "global_batch": w.B * args.gpus, "seq_len": w.T,
             "parallelism": f"dp{args.gpus}", "l2": "inputs 17 GB > 129 MB L2: no flush"}
 
 
@@ -236,6 +237,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--fit-every", type=int, default=1)
+    ap.add_argument("--alloc-mode", type=int, default=0,
+                    help="0: widths from the previous write-back's statistics; 1: from this one's")
     ap.add_argument("--T", type=int, default=None, help="tokens per step (default: workload T)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
@@ -261,7 +264,7 @@ def main():
     torch.cuda.set_device(dev)
     q.load(build_if_missing=True)
 
-    cfg = q.Config.from_workload(w, fit_every=args.fit_every)
+    cfg = q.Config.from_workload(w, fit_every=args.fit_every, alloc_mode=args.alloc_mode)
     x = synth.device_inputs(w, device=dev, seed_offset=rank_seed_offset(rank))
     nchan = w.H * w.dk
     L = 1 << w.gate_bits
@@ -365,7 +368,9 @@ def main():
                "staging": f"qstate_scan_host, {chunk}-token chunks on a copy stream"}
         q.qstate_check(comp)
 
-    launches_per_step = 4 + 2 + 2 * w.T   # decay (4), init (alloc + pack), T x (write-back + alloc)
+    # decay quantiser (4), init (alloc + pack), then per write-back: write-back + alloc, or with
+    # current-statistics allocation a statistics pass + alloc + write-back
+    launches_per_step = 4 + 2 + (3 if args.alloc_mode == 1 else 2) * w.T
     clocks = clk.summary()
     if rank != 0:
         if world > 1:

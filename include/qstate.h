@@ -51,6 +51,15 @@ extern "C" {
 #define QSTATE_ERASE_GENERAL 2 /* a and w given per token (Eq. 1 in general)                  */
 #define QSTATE_UNIT_ROW 0    /* width + FP16 scale per row (Sec. 3, "Allocation units")       */
 #define QSTATE_UNIT_HEAD 1   /* width per head, FP16 scale per 32 key rows x value column     */
+/* When the allocation of Eq. 3-4 sees its statistics.  LAGGED: the widths a write-back
+ * packs with were allocated from the statistics after the previous write-back (qstate_step
+ * allocates into `in` after writing `out`).  CURRENT: qstate_step first runs the interval's
+ * tokens to get this write-back's ranges and EMAs, allocates from them into out->widths /
+ * out->head_off, then packs with those widths (the state and the tokens are processed twice);
+ * row unit only. */
+#define QSTATE_ALLOC_LAGGED 0
+#define QSTATE_ALLOC_CURRENT 1
+
 /* Allocation weights c_i (Eq. 3 and the alternatives of Table 1).  With the EMAs of
  * qstate_stats, m_s = EMA(1 - e^{-2s}) and m_r = EMA of the erasure term:
  * Gamma_hat = (1 - m_s) / (expm1(m_r) + m_s); Rtilde^2 = R^2 / mean of R^2 over the unit's
@@ -87,6 +96,7 @@ typedef struct qstate_cfg {
     float ema_span;              /* EMA span in tokens (Sec. 3: 64)                           */
     int32_t gate_bits;           /* 0: FP32 decay rates; g in 1..8: log-quantised rates       */
     int32_t weight_kind;         /* QSTATE_WEIGHT_*                                          */
+    int32_t alloc_mode;          /* QSTATE_ALLOC_LAGGED (0) or QSTATE_ALLOC_CURRENT (1)       */
 } qstate_cfg;
 
 /* One packed state (device pointers).  Layout (Sec. 3, "Levels and storage"; bit order is

@@ -41,7 +41,7 @@ class OrcCfg(ct.Structure):
                 ("bbar_num", ct.c_int32), ("bbar_den", ct.c_int32), ("bmin", ct.c_int32),
                 ("bmax", ct.c_int32), ("C", ct.c_int32), ("fit_every", ct.c_int32),
                 ("ema_span", ct.c_float), ("gate_bits", ct.c_int32),
-                ("weight_kind", ct.c_int32)]
+                ("weight_kind", ct.c_int32), ("alloc_mode", ct.c_int32)]
 
 
 @dataclass
@@ -64,6 +64,7 @@ class Cfg:
     ema_span: float = 64.0
     gate_bits: int = 0
     weight_kind: int = 0
+    alloc_mode: int = 0      # 0 lagged widths, 1 widths from this write-back's statistics
 
     def c(self) -> OrcCfg:
         return OrcCfg(*[getattr(self, f) for f, _ in OrcCfg._fields_])
@@ -123,6 +124,7 @@ def lib():
         L.orc_init_widths.argtypes = [ct.POINTER(OrcCfg), P, P]
         L.orc_quant_decay.argtypes = [ct.c_long, ct.c_int, P, ct.c_int, P, P, P]
         L.orc_step.argtypes = ([ct.POINTER(OrcCfg)] + [P] * 10 + [ct.c_int] * 4 + [P] * 14)
+        L.orc_step_current.argtypes = ([ct.POINTER(OrcCfg)] + [P] * 10 + [ct.c_int] * 4 + [P] * 14)
     return _lib
 
 
@@ -370,7 +372,8 @@ def step(cfg: Cfg, src: Buf, dst: Buf, inp: dict, t_begin, t_end, w_index, o, em
     w_in = _c(inp["w"], np.float32) if "w" in inp else None
     sc = None if s_code is None else _c(s_code, np.uint8)
     sl = None if s_lut is None else _c(s_lut, np.float32)
-    rc = lib().orc_step(ct.byref(c), _p(src.payload), _p(src.scales), _p(src.widths),
+    fn = lib().orc_step_current if cfg.alloc_mode == 1 else lib().orc_step
+    rc = fn(ct.byref(c), _p(src.payload), _p(src.scales), _p(src.widths),
                         _p(src.head_off), _p(src.fidx), _p(dst.payload), _p(dst.scales),
                         _p(dst.widths), _p(dst.head_off), _p(dst.fidx), T, t_begin, t_end,
                         w_index, _p(q), _p(k), _p(v), _p(s), _p(sc), _p(sl), _p(beta), _p(o),
@@ -392,7 +395,8 @@ def scan(cfg: Cfg, inp: dict, T=None, s_code=None, s_lut=None):
     for t0 in range(0, T, cfg.C):
         t1 = min(T, t0 + cfg.C)
         step(cfg, src, dst, inp, t0, t1, w, o, ema_s, ema_r, rng, s_code, s_lut)
-        src.widths[:], src.head_off[:] = alloc(cfg, ema_s, ema_r, rng)
+        if cfg.alloc_mode == 0:   # lagged: the next write-back packs with widths from these statistics
+            src.widths[:], src.head_off[:] = alloc(cfg, ema_s, ema_r, rng)
         src, dst = dst, src
         w += 1
     return o, src, ema_s, ema_r, rng

@@ -37,6 +37,8 @@ typedef struct {
     float ema_span;      /* 64 tokens                                                         */
     int32_t gate_bits;   /* 0: FP32 rates; g > 0: log-quantised rates                         */
     int32_t weight_kind; /* 0: c = Gamma_hat * Rtilde^2 (Eq. 3)                                */
+    int32_t alloc_mode;  /* 0: widths from the previous write-back's statistics (lagged);
+                            1: widths from this write-back's statistics (orc_step_current)  */
 } orc_cfg;
 
 #define ORC_OK 0
@@ -824,4 +826,51 @@ int orc_step(const orc_cfg* c, const uint8_t* pay_in, const uint16_t* sc_in, con
     free(d);
     free(p);
     return ORC_OK;
+}
+
+/* ---------------------------------------------------------------------------------------
+ * One write-back with the allocation taken from this write-back's own statistics (the
+ * reading of Eq. 3 that uses the ranges of the state being quantised; Sec. 3):
+ *   1. run the interval's tokens for every head (orc_step into scratch buffers laid out like
+ *      the input), which updates the EMAs and ranges and writes the readouts;
+ *   2. allocate widths and head offsets from those statistics (orc_alloc) into w_out/off_out;
+ *   3. quantise + pack every head's state with the new widths.
+ * ------------------------------------------------------------------------------------- */
+int orc_step_current(const orc_cfg* c, const uint8_t* pay_in, const uint16_t* sc_in,
+                     const uint8_t* w_in, const uint32_t* off_in, const uint8_t* fidx_in,
+                     uint8_t* pay_out, uint16_t* sc_out, uint8_t* w_out, uint32_t* off_out,
+                     uint8_t* fidx_out, int T, int t_begin, int t_end, int w_index,
+                     const float* q, const float* k, const float* v, const float* s,
+                     const uint8_t* s_code, const float* s_lut, const float* beta, float* o,
+                     float* ema_s, float* ema_r, float* range, float* x_dump,
+                     const float* a_tok, const float* w_tok) {
+    if (c->unit_kind != 0) return ORC_EINVAL;
+    int H = c->H, dk = c->dk, dv = c->dv;
+    long rb = orc_region_bytes(c);
+    if (rb < 0) return ORC_EINVAL;
+    size_t n_el = (size_t)c->B * H * dk * dv, n_sc = (size_t)c->B * H * dk;
+    float* X = (float*)malloc(sizeof(float) * n_el);
+    uint8_t* pay_tmp = (uint8_t*)malloc((size_t)c->B * rb);
+    uint16_t* sc_tmp = (uint16_t*)malloc(sizeof(uint16_t) * n_sc);
+    uint8_t* fidx_tmp = (uint8_t*)malloc(n_sc);
+    int rc = orc_step(c, pay_in, sc_in, w_in, off_in, fidx_in, pay_tmp, sc_tmp, w_in, off_in,
+                      fidx_tmp, T, t_begin, t_end, w_index, q, k, v, s, s_code, s_lut, beta, o,
+                      ema_s, ema_r, range, X, a_tok, w_tok);
+    if (rc == ORC_OK) rc = orc_alloc(c, ema_s, ema_r, range, w_out, off_out);
+    if (rc == ORC_OK && !layout_ok(c, w_out, off_out)) rc = ORC_EINVAL;
+    if (rc == ORC_OK) {
+        memset(pay_out, 0, (size_t)c->B * rb);
+        for (int b = 0; b < c->B; b++)
+            for (int h = 0; h < H; h++) {
+                int refit = (c->fit_every <= 1) || ((w_index + h) % c->fit_every == 0);
+                pack_head(c, b, h, X + ((size_t)b * H + h) * dk * dv, w_out, off_out, refit,
+                          fidx_in, pay_out, sc_out, fidx_out, range);
+            }
+        if (x_dump) memcpy(x_dump, X, sizeof(float) * n_el);
+    }
+    free(X);
+    free(pay_tmp);
+    free(sc_tmp);
+    free(fidx_tmp);
+    return rc;
 }

@@ -96,6 +96,10 @@ int validate(const qstate_cfg* c) {
     if (c->fit_every < 1) return fail(QSTATE_EINVAL, "fit_every must be >= 1");
     if (!(c->ema_span > 0.0f)) return fail(QSTATE_EINVAL, "ema_span must be > 0");
     if (c->gate_bits < 0 || c->gate_bits > 8) return fail(QSTATE_EINVAL, "gate_bits must be in [0, 8]");
+    if (c->alloc_mode != QSTATE_ALLOC_LAGGED && c->alloc_mode != QSTATE_ALLOC_CURRENT)
+        return fail(QSTATE_EINVAL, "unsupported alloc_mode %d", c->alloc_mode);
+    if (c->alloc_mode == QSTATE_ALLOC_CURRENT && c->unit_kind != QSTATE_UNIT_ROW)
+        return fail(QSTATE_EINVAL, "alloc_mode current is for the row unit");
     if (c->weight_kind < QSTATE_WEIGHT_OURS || c->weight_kind > QSTATE_WEIGHT_UNIFORM)
         return fail(QSTATE_EINVAL, "unsupported weight_kind %d", c->weight_kind);
     return QSTATE_OK;
@@ -410,6 +414,19 @@ int qstate_step(const qstate_cfg* cfg, qstate_buf* in, qstate_buf* out, const qs
     p.ema_s = stats->ema_s;
     p.ema_r = stats->ema_r;
     p.range = stats->range;
+    if (cfg->alloc_mode == QSTATE_ALLOC_CURRENT) {
+        // this write-back's statistics, the allocation from them, then the write-back proper
+        if (!wb_row_eligible(*cfg, p))
+            return fail(QSTATE_EINVAL, "alloc_mode current needs 16-byte aligned buffers and fidx");
+        p.mode = 1;
+        if ((e = launch_writeback(*cfg, p, st)) != cudaSuccess) return cuda_fail(e, "statistics pass");
+        rc = run_alloc(cfg, stats->ema_s, stats->ema_r, stats->range, 0, out->widths,
+                       out->head_off, status, st);
+        if (rc) return rc;
+        p.mode = 2;
+        if ((e = launch_writeback(*cfg, p, st)) != cudaSuccess) return cuda_fail(e, "write-back kernel");
+        return QSTATE_OK;
+    }
     e = launch_writeback(*cfg, p, st);
     if (e != cudaSuccess) return cuda_fail(e, "write-back kernel");
     return run_alloc(cfg, stats->ema_s, stats->ema_r, stats->range, 0, in->widths, in->head_off,

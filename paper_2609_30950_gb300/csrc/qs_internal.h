@@ -23,6 +23,8 @@ struct StepParams {
     int t_begin, t_end, w_index;
     int erase;        // 1: delta rule (a = beta k, w = beta 1); 0: a = 0, w = 1 (or general)
     int general;      // 1: a and w given per token (a_in, w_in)
+    int mode;         // 0: full write-back; 1: statistics only (ranges, EMAs, readouts; no
+                      // packing); 2: full write-back leaving the EMAs in memory unchanged
     int decay_row;    // 1: per-row rates; 0: per-head rates
     int fit_every;
     int L;            // 2^gate_bits (0 when rates are FP32)

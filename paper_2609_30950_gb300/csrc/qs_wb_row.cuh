@@ -434,7 +434,7 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
 #pragma unroll
             for (int jj = 0; jj < PER; ++jj) {
                 const int w = wa[lane * PER + jj];
-                bad |= (w > 16);
+                bad |= (w > 16) && (warp == 0 || p.mode != 1);   // statistics only: no output rows
                 loc[jj] = sum;
                 sum += w * (DV / 8);
             }
@@ -452,8 +452,9 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                 off[DK] = total;
                 const int align = DV == 128 ? 16 : 8;
                 if (warp == 0) bad |= (total != S.in_end - S.in_off);
-                else bad |= (total > p.stage_bytes || S.out_off % align != 0 || S.out_off < 0 ||
-                             static_cast<long long>(S.out_off) + total > p.region_bytes);
+                else if (p.mode != 1)
+                    bad |= (total > p.stage_bytes || S.out_off % align != 0 || S.out_off < 0 ||
+                            static_cast<long long>(S.out_off) + total > p.region_bytes);
                 if (bad) atomicExch(&sm.flag, 1);
             }
         } else if (tid >= 64 && tid < 64 + DK) {
@@ -711,6 +712,10 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
             float R = lmax;
 #pragma unroll
             for (int o = 1; o < TPR; o <<= 1) R = fmaxf(R, __shfl_xor_sync(kFull, R, o));
+            if (p.mode == 1) {   // statistics only: the range is all this pass produces
+                if (q == 0) sm.rowR[i] = R;
+                continue;
+            }
             float D = 0.0f;
             int fidx = S.fidx[i];
             if (__any_sync(kFull, w == 1)) {
@@ -806,10 +811,12 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
         // ---- stores -------------------------------------------------------------------------------
         const size_t rb = static_cast<size_t>(g) * DK;
         if (tid < DK) {
-            p.out_scales[rb + tid] = sm.out_scale[tid];
-            p.out_fidx[rb + tid] = sm.out_fidx[tid];
+            if (p.mode != 1) {
+                p.out_scales[rb + tid] = sm.out_scale[tid];
+                p.out_fidx[rb + tid] = sm.out_fidx[tid];
+            }
             if (p.range) p.range[rb + tid] = sm.rowR[tid];
-            if (stats) {
+            if (stats && p.mode != 2) {
                 p.ema_s[rb + tid] = S.ms[tid];
                 p.ema_r[rb + tid] = S.mr[tid];
             }

@@ -47,6 +47,8 @@ class Workload:
     gate_bits: int = 0        # 0: FP32 decay rates; g > 0: log-quantised rates with 2**g levels
     s_loc: float = -2.0       # decay rate s = softplus(N(s_loc, 1))
     kq_std: float = 0.0       # 0: unit-norm Gaussian keys/queries; > 0: N(0, kq_std^2) entries
+    persistent: float = 0.0   # > 0: per-channel decay fixed over tokens, log-uniform over
+                              # [persistent, 1] (slow channels that keep their rate)
     seed: int = 0
     notes: str = field(default="", compare=False)
 
@@ -87,6 +89,11 @@ EXTENSION_WORKLOADS = {
                             bmin=1, bmax=8, unit="row", seed=5000),
     "gdn_general": Workload("gdn_general", GDN_GEN, B=16, H=16, dk=128, dv=128, T=256, C=1, bbar=4,
                             bmin=2, bmax=16, unit="head", s_loc=-3.0, seed=6000),
+    # KDA with persistent per-channel decay: each (b, h, i) keeps one rate over all tokens,
+    # log-uniform in [1e-3, 1] (slow channels accumulate errors across write-backs)
+    "kda_persistent": Workload("kda_persistent", KDA, B=32, H=8, dk=128, dv=128, T=256, C=1,
+                               bbar=4, bmin=0, bmax=8, unit="row", gate_bits=2, persistent=1e-3,
+                               seed=7000),
 }
 
 
@@ -147,7 +154,11 @@ def host_inputs(w: Workload, b_range=None, t_range=None) -> dict:
             k[bi, ti] = _keys(_rng(w.seed, _K, b, t), H, dk, w.kq_std)
             v[bi, ti] = _rng(w.seed, _V, b, t).standard_normal((H, dv))
             shape = (H, dk) if w.per_row_decay else (H,)
-            s[bi, ti] = _softplus(w.s_loc + _rng(w.seed, _S, b, t).standard_normal(shape))
+            if w.persistent > 0:   # one draw per (b, channel), the same for every token
+                u = _rng(w.seed, _S, b, 0).uniform(size=shape)
+                s[bi, ti] = np.exp(np.log(w.persistent) * (1.0 - u))
+            else:
+                s[bi, ti] = _softplus(w.s_loc + _rng(w.seed, _S, b, t).standard_normal(shape))
             beta[bi, ti] = _sigmoid(_rng(w.seed, _BETA, b, t).standard_normal((H,)))
             if w.general:
                 g = _rng(w.seed, _A, b, t).standard_normal((H, dk)) / np.sqrt(dk)
@@ -178,7 +189,11 @@ def device_inputs(w: Workload, device="cuda", T=None, seed_offset=0):
     k = keys(dk)
     v = torch.randn((B, T, H, dv), **f32)
     shape = (B, T, H, dk) if w.per_row_decay else (B, T, H)
-    s = torch.nn.functional.softplus(torch.randn(shape, **f32).add_(w.s_loc))
+    if w.persistent > 0:
+        u = torch.rand((B, 1) + shape[2:], **f32)
+        s = torch.exp(u.neg_().add_(1.0).mul_(float(np.log(w.persistent)))).expand(shape).contiguous()
+    else:
+        s = torch.nn.functional.softplus(torch.randn(shape, **f32).add_(w.s_loc))
     beta = torch.sigmoid(torch.randn((B, T, H), **f32))
     out = dict(q=q, k=k, v=v, s=s, beta=beta)
     if w.general:

@@ -322,6 +322,55 @@ def test_quantised_lockstep_fit_every(qs, orc):
     _lockstep(qs, orc, w, fit_every=4)
 
 
+def test_persistent_decay_lockstep(qs, orc):
+    """KDA with per-channel decay fixed over tokens (slow channels, log-quantised rates)."""
+    w = synth.scaled(synth.EXTENSION_WORKLOADS["kda_persistent"], B=3, H=4, T=12)
+    _lockstep(qs, orc, w, log_decay=True)
+
+
+@pytest.mark.parametrize("name,log_decay", [("kda_decode", True), ("mamba2_decode", False),
+                                            ("kda_prefill", False)])
+def test_current_allocation_lockstep(qs, orc, name, log_decay):
+    """alloc_mode current: each write-back allocates from its own statistics (a statistics
+    pass, the allocation, then the packing pass).  The oracle runs free; before every
+    write-back its state is copied into the GPU; widths, codes, readouts and statistics of the
+    GPU's write-back are compared with the oracle's."""
+    w = SMALL[name]
+    cfgq = qs.Config.from_workload(w, alloc_mode=1)
+    cfgo = orc.Cfg.from_workload(w, alloc_mode=1)
+    inp = synth.host_inputs(w)
+    s_code = s_lut = None
+    if log_decay:
+        nchan = w.H * w.dk if w.per_row_decay else w.H
+        s_code, s_lut, _ = orc.quant_decay(inp["s"], nchan, w.gate_bits)
+    X, _ = _dev_inputs(w, inp, qs, s_code, s_lut)
+    src, dst = orc.init_state(cfgo)
+    z = lambda: np.zeros(cfgo.B * cfgo.units, np.float32)
+    ms, mr, R = z(), z(), z()
+    oo = np.zeros((w.B, w.T, w.H, w.dv), np.float32)
+    A, Bst = qs.new_state(cfgq), qs.new_state(cfgq)
+    qs.qstate_init(cfgq, A, Bst)
+    gst = qs.new_stats(cfgq)
+    o = torch.zeros((w.B, w.T, w.H, w.dv), dtype=torch.float32, device="cuda")
+    for wi, t0 in enumerate(range(0, w.T, w.C)):
+        t1 = min(w.T, t0 + w.C)
+        gsrc, gdst = (A, Bst) if wi % 2 == 0 else (Bst, A)
+        set_gpu_state(gsrc, src)
+        for t, a in zip((gst.ema_s, gst.ema_r, gst.range), (ms, mr, R)):
+            t.copy_(torch.from_numpy(a).cuda())
+        qs.qstate_step(cfgq, gsrc, gdst, X, t0, t1, wi, o, gst)
+        qs.qstate_check()
+        xo = orc.step(cfgo, src, dst, inp, t0, t1, wi, oo, ms, mr, R, s_code, s_lut, want_x=True)
+        g_out = from_gpu_state(orc, gdst)
+        assert np.array_equal(g_out.widths, dst.widths), wi      # allocated from this write-back
+        assert np.array_equal(g_out.head_off, dst.head_off), wi
+        compare_packed(orc, cfgo, g_out, dst, X=xo)
+        assert rel_err_vectors(host(o, np.float32)[:, t0:t1], oo[:, t0:t1]) <= REL_O_QUANT
+        for g, r in ((gst.ema_s, ms), (gst.ema_r, mr), (gst.range, R)):
+            assert np.allclose(host(g, np.float32), r, rtol=REL_STATS, atol=1e-30), wi
+        src, dst = dst, src
+
+
 @pytest.mark.parametrize("name", ["kda_general", "gdn_general"])
 def test_general_erasure_lockstep(qs, orc, name):
     """Eq. (1) with a and w given per token (row unit and head unit) stays in lockstep."""

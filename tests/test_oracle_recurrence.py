@@ -297,3 +297,42 @@ def test_general_erasure_needs_a_and_w(orc):
     z = lambda: np.zeros(cfg.B * cfg.units, np.float32)
     with pytest.raises(ValueError):
         orc.step(cfg, src, dst, synth.host_inputs(w), 0, 1, 0, o, z(), z(), z())
+
+
+def test_current_allocation_uses_this_write_backs_statistics(orc):
+    """alloc_mode 1: the widths a write-back packs with are the allocation of the statistics
+    that write-back produced (its own ranges and EMAs), and the budget still holds; with
+    alloc_mode 0 they are those of the previous write-back."""
+    w = _small("kda_decode", B=2, H=3, T=5, gate_bits=0)
+    for mode in (0, 1):
+        cfg = orc.Cfg.from_workload(w, alloc_mode=mode)
+        inp = synth.host_inputs(w)
+        src, dst = orc.init_state(cfg)
+        o = np.zeros((w.B, w.T, w.H, w.dv), np.float32)
+        ms, mr, R = (np.zeros(cfg.B * cfg.units, np.float32) for _ in range(3))
+        for t in range(w.T):
+            before = orc.alloc(cfg, ms, mr, R)[0] if t else None
+            orc.step(cfg, src, dst, inp, t, t + 1, t, o, ms, mr, R)
+            now = orc.alloc(cfg, ms, mr, R)[0]
+            if mode == 1:
+                assert np.array_equal(dst.widths, now)
+            elif t:
+                assert np.array_equal(dst.widths, before)
+            assert dst.widths.reshape(w.B, -1).sum(axis=1).tolist() == [cfg.units * 4] * w.B
+            if mode == 0:
+                src.widths[:], src.head_off[:] = orc.alloc(cfg, ms, mr, R)
+            src, dst = dst, src
+
+
+def test_current_allocation_tracks_ranges_better_at_low_bits(orc):
+    """Widths from the current ranges follow the state being quantised; on a two-bit budget
+    they give a readout error no worse than lagged widths over a short scan."""
+    w = _small("tiny_kda", T=96, bbar=2, bmin=1, bmax=8)
+    inp = synth.host_inputs(w)
+    ref, _ = orc.recur(np.zeros((w.dk, w.dv)), *orc.expand_inputs(orc.Cfg.from_workload(w), inp, 0, 0),
+                       dtype=np.float64)
+    err = {}
+    for mode in (0, 1):
+        o, *_ = orc.scan(orc.Cfg.from_workload(w, alloc_mode=mode), inp)
+        err[mode] = float(np.mean((o[0, :, 0] - ref) ** 2) / np.mean(ref ** 2))
+    assert err[1] <= 1.05 * err[0], err
