@@ -236,7 +236,7 @@ int qstate_scan(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong,
 /* qstate_scan fed from pinned host memory, for callers whose token inputs and readouts live
  * on the host.  x_host and x_dev describe the same (B, T, H, .) tensors (same T) in host and
  * device memory; every input present in x_host (q, k, v, beta, s or s_code) is copied, token
- * chunk by token chunk, into x_dev's buffer with one 2D copy per tensor and chunk on
+ * chunk by token chunk, into x_dev's buffer (one copy per tensor, chunk and batch element) on
  * copy_stream, while the compute stream runs the scan of the previous chunk; inputs absent
  * from x_host (e.g. rate codes made on the device by qstate_quant_decay) must already be in
  * x_dev.  Readouts of each chunk are copied from o_dev to o_host on copy_stream once the chunk

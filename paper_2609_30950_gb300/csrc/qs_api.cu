@@ -189,6 +189,22 @@ void set_inputs(StepParams& p, const qstate_inputs* x) {
     p.w_in = x->w;
 }
 
+// Staging of token chunks between pinned host memory and the device: tokens [t0, t1) of every
+// batch element of a (B, T, per-token bytes) tensor, 16 bytes per thread and step.  The host
+// side is read or written in place (pinned memory is mapped into the device address space), so
+// one small launch replaces B row copies; it needs few registers and no shared memory and so
+// shares SMs with the write-back kernel.
+__global__ void __launch_bounds__(128) stage_tokens_kernel(uint4* dst, const uint4* src, int B,
+                                                           long long pitch16, long long off16,
+                                                           long long width16) {
+    const long long n = static_cast<long long>(B) * width16;
+    for (long long e = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x; e < n;
+         e += static_cast<long long>(gridDim.x) * blockDim.x) {
+        const long long b = e / width16, c = e - b * width16;
+        dst[b * pitch16 + off16 + c] = src[b * pitch16 + off16 + c];
+    }
+}
+
 // The shuffled-decay bijection of N units: u -> (A u + N / 3) mod N with A the smallest
 // integer above 0.6180339887 N that is coprime to N.
 int gcd_int(int a, int b) { return b == 0 ? a : gcd_int(b, a % b); }
@@ -484,11 +500,28 @@ int qstate_scan_host(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong,
                         {(void*)x_dev->v, x_host->v, H * cfg->dv * f4}, {(void*)x_dev->beta, x_host->beta, H * f4},
                         {(void*)x_dev->s, x_host->s, nchan * f4}, {(void*)x_dev->s_code, x_host->s_code, nchan},
                         {(void*)x_dev->a, x_host->a, H * cfg->dk * f4}, {(void*)x_dev->w, x_host->w, H * cfg->dv * f4}};
-    // tokens [t0, t1) of a (B, T, per) token-major tensor: one 2D copy, rows = batch elements
+    // tokens [t0, t1) of a (B, T, per) token-major tensor: one copy per batch element (one
+    // copy in all when the chunk spans every token); plain copies move pinned host memory at
+    // full link speed where strided 2D copies were measured several times slower
     auto copy_tokens = [&](void* dst, const void* src, size_t per, int t0, int t1, cudaMemcpyKind kind) {
         const size_t pitch = static_cast<size_t>(T) * per, off = static_cast<size_t>(t0) * per;
-        return cudaMemcpy2DAsync(static_cast<char*>(dst) + off, pitch, static_cast<const char*>(src) + off,
-                                 pitch, static_cast<size_t>(t1 - t0) * per, B, kind, ts);
+        const size_t width = static_cast<size_t>(t1 - t0) * per;
+        if (width == pitch)
+            return cudaMemcpyAsync(dst, src, pitch * B, kind, ts);
+        const bool a16 = per % 16 == 0 && (reinterpret_cast<uintptr_t>(dst) & 15) == 0 &&
+                         (reinterpret_cast<uintptr_t>(src) & 15) == 0;
+        if (a16) {
+            stage_tokens_kernel<<<2 * 152, 128, 0, ts>>>(static_cast<uint4*>(dst), static_cast<const uint4*>(src),
+                                                        B, static_cast<long long>(pitch / 16),
+                                                        static_cast<long long>(off / 16),
+                                                        static_cast<long long>(width / 16));
+            return cudaGetLastError();
+        }
+        cudaError_t err = cudaSuccess;
+        for (int bb = 0; bb < B && err == cudaSuccess; ++bb)
+            err = cudaMemcpyAsync(static_cast<char*>(dst) + bb * pitch + off,
+                                  static_cast<const char*>(src) + bb * pitch + off, width, kind, ts);
+        return err;
     };
     qstate_buf* src = ping;
     qstate_buf* dst = pong;
