@@ -8,6 +8,10 @@ allocation for the next one.  Inputs (17 GB) are resident in HBM when the timed 
 and exceed L2, so no flush is needed.  Prints one JSON line.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference] [--fit-every F]
+                    [--workload gdn_decode|mamba2_decode|kda_prefill|...]
+
+``--workload`` runs another of the paper's layer shapes (a labelled secondary measurement);
+the default is KDA decode.
 
 Under torchrun each rank runs the same per-GPU batch (batch elements are independent: weak
 scaling, no collective); the reported value is the sum over ranks divided by the slowest rank.
@@ -34,24 +38,32 @@ PEAK_FALLBACK_GBS = 6800.0
 
 
 def algorithmic_bytes(w, fit_every=1):
-    """Bytes the method must move per write-back launch (the fused kernel) and per allocation
-    launch, itemised per head for the row unit with log-coded rates:
+    """Bytes the method must move per write-back launch (the fused kernel, C tokens) and per
+    allocation launch.  Per head, with u units and g scale groups per head (row unit: u = g =
+    dk; head unit: u = 1, g = dk dv / 32):
       payload read + write        2 dk dv bbar / 8
-      FP16 scales read + write    2 * 2 dk
-      widths read (in + out)      2 dk
-      fitted-factor index r + w   2 dk
+      FP16 scales read + write    2 * 2 g
+      widths read (in + out)      2 u
+      fitted-factor index r + w   2 g
       head offsets (in + out)     8
-      EMA statistics r + w        2 * 2 * 4 dk
-      row range write             4 dk
+      EMA statistics r + w        2 * 2 * 4 u
+      range write                 4 u
+    and per token
       q, k, v                     4 (2 dk + dv)
-      rate codes + beta           dk + 4
+      decay rates                 dk (row, log-coded), 4 dk (row, FP32), 4 (head)
+      beta                        4 (delta rule)
       readout o                   4 dv
-    Allocation per batch element: EMA + range read 12 per row, widths 1 per row, offsets 4 H."""
+    Allocation per batch element: EMA + range read 12 per unit, widths 1 per unit, offsets 4 H."""
     dk, dv = w.dk, w.dv
-    per_head = (2 * dk * dv * w.bbar // 8 + 4 * dk + 2 * dk + 2 * dk + 8 + 16 * dk + 4 * dk +
-                4 * (2 * dk + dv) + (dk if w.gate_bits else 4 * dk) + 4 + 4 * dv)
+    row = w.unit == "row"
+    u = dk if row else 1
+    g = dk if row else dk * dv // 32
+    rates = (dk if w.gate_bits else 4 * dk) if w.per_row_decay else 4
+    per_token = 4 * (2 * dk + dv) + rates + (4 if w.erase else 0) + 4 * dv
+    per_head = (2 * dk * dv * w.bbar // 8 + 4 * g + 2 * u + 2 * g + 8 + 16 * u + 4 * u +
+                w.C * per_token)
     writeback = per_head * w.B * w.H
-    alloc = w.B * (w.H * dk * 13 + 4 * w.H)
+    alloc = w.B * (w.H * u * 13 + 4 * w.H)
     return writeback, alloc, per_head
 
 
@@ -146,28 +158,30 @@ class ClockSampler:
 
 def cpu_baseline(w, budget_s=12.0):
     """The oracle as it stands, single-threaded, on a bounded sample of the workload: the
-    log-decay quantiser over the sample's rates, then per token one write-back of every head
-    of the sampled batch elements and the allocation.  Returns tokens/s and the sample."""
+    log-decay quantiser over the sample's rates (when rates are coded), then per write-back one
+    pass over every head of the sampled batch elements and the allocation.  Returns tokens/s
+    and the sample."""
     import numpy as np
     from oracle import oracle as orc
-    nb, nt = 4, 64
+    nb, nt = 4, max(64, w.C)
     sub = synth.scaled(w, B=nb)
     cfg = orc.Cfg.from_workload(sub)
     t_start = time.perf_counter()
     inp = synth.host_inputs(sub, t_range=(0, nt))
     gen_s = time.perf_counter() - t_start
     t0 = time.perf_counter()
-    nchan = w.H * w.dk
-    codes, lut, _ = orc.quant_decay(inp["s"], nchan, w.gate_bits)
+    codes = lut = None
+    if w.gate_bits:
+        codes, lut, _ = orc.quant_decay(inp["s"], w.H * w.dk, w.gate_bits)
     src, dst = orc.init_state(cfg)
     o = np.zeros((nb, nt, w.H, w.dv), np.float32)
     ms, mr, R = (np.zeros(cfg.units * nb, np.float32) for _ in range(3))
     tokens = 0
-    for t in range(nt):
-        orc.step(cfg, src, dst, inp, t, t + 1, t, o, ms, mr, R, codes, lut)
+    for wi, t in enumerate(range(0, nt, w.C)):
+        orc.step(cfg, src, dst, inp, t, t + w.C, wi, o, ms, mr, R, codes, lut)
         src.widths[:], src.head_off[:] = orc.alloc(cfg, ms, mr, R)
         src, dst = dst, src
-        tokens += nb
+        tokens += nb * w.C
         if time.perf_counter() - t0 > budget_s:
             break
     el = time.perf_counter() - t0
@@ -227,7 +241,15 @@ def config_of(w, args):
             "bbar": w.bbar, "widths": [w.bmin, w.bmax], "gate_bits": w.gate_bits,
             "fit_every": args.fit_every, "alloc_mode": getattr(args, "alloc_mode", 0),
             "global_batch": w.B * args.gpus, "seq_len": w.T,
-            "parallelism": f"dp{args.gpus}", "l2": "inputs 17 GB > 129 MB L2: no flush"}
+            "parallelism": f"dp{args.gpus}",
+            "l2": (f"inputs {input_gb(w):.1f} GB > 129 MB L2: no flush" if input_gb(w) > 0.129
+                   else f"inputs {input_gb(w) * 1e3:.1f} MB fit in L2 (small case)")}
+
+
+def input_gb(w):
+    """Token inputs of one step (q, k, v, FP32 rates, beta), which each step streams through."""
+    rates = w.dk if w.per_row_decay else 1
+    return w.B * w.T * w.H * (2 * w.dk + w.dv + rates + 1) * 4 / 1e9
 
 
 def main():
@@ -242,9 +264,11 @@ def main():
     ap.add_argument("--T", type=int, default=None, help="tokens per step (default: workload T)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--workload", default=WORKLOAD, choices=sorted(synth.WORKLOADS),
+                    help="the paper's layer shape to run (default: KDA decode)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
-    w = synth.WORKLOADS[WORKLOAD]
+    w = synth.WORKLOADS[args.workload]
     if args.T:
         w = synth.scaled(w, T=args.T)
     if args.impl == "reference":
@@ -267,18 +291,26 @@ def main():
     cfg = q.Config.from_workload(w, fit_every=args.fit_every, alloc_mode=args.alloc_mode)
     x = synth.device_inputs(w, device=dev, seed_offset=rank_seed_offset(rank))
     nchan = w.H * w.dk
-    L = 1 << w.gate_bits
-    codes = torch.empty(x["s"].shape, dtype=torch.uint8, device=dev)
-    lut = torch.empty(nchan * L, dtype=torch.float32, device=dev)
-    thr = torch.empty(nchan * (L - 1), dtype=torch.float32, device=dev)
+    coded = w.gate_bits > 0
+    codes = lut = thr = None
+    if coded:
+        L = 1 << w.gate_bits
+        codes = torch.empty(x["s"].shape, dtype=torch.uint8, device=dev)
+        lut = torch.empty(nchan * L, dtype=torch.float32, device=dev)
+        thr = torch.empty(nchan * (L - 1), dtype=torch.float32, device=dev)
+    beta = x["beta"] if w.erase else None
     o = torch.empty((w.B, w.T, w.H, w.dv), dtype=torch.float32, device=dev)
     A, Bst = q.new_state(cfg, dev), q.new_state(cfg, dev)
     st = q.new_stats(cfg, dev)
-    X = q.Inputs(x["q"], x["k"], x["v"], None, codes, lut, x["beta"], w.T)
+    X = q.Inputs(x["q"], x["k"], x["v"], None if coded else x["s"], codes, lut, beta, w.T)
     stream = torch.cuda.current_stream(dev)
 
+    def quant_decay(s):
+        if coded:
+            q.qstate_quant_decay(cfg, x["s"], codes, lut, thr, s)
+
     def step():
-        q.qstate_quant_decay(cfg, x["s"], codes, lut, thr, stream)
+        quant_decay(stream)
         q.qstate_init(cfg, A, Bst, stream)
         q.qstate_scan(cfg, A, Bst, X, 0, w.T, 0, o, st, stream)
 
@@ -303,7 +335,7 @@ def main():
         start.record(stream)
         for e0, e1, e2 in ev:
             e0.record(stream)
-            q.qstate_quant_decay(cfg, x["s"], codes, lut, thr, stream)
+            quant_decay(stream)
             q.qstate_init(cfg, A, Bst, stream)
             e1.record(stream)
             q.qstate_scan(cfg, A, Bst, X, 0, w.T, 0, o, st, stream)
@@ -318,7 +350,8 @@ def main():
     value = job_throughput(tokens_step, world, ms_step)
     scan_ms = statistics.median(e1.elapsed_time(e2) for _, e1, e2 in ev)
     decay_ms = statistics.median(e0.elapsed_time(e1) for e0, e1, _ in ev)
-    per_wb_ms = scan_ms / w.T        # write-back kernel + allocation kernel per token
+    n_wb = -(-w.T // w.C)
+    per_wb_ms = scan_ms / n_wb       # write-back kernel + allocation kernel per write-back
 
     wb_bytes, alloc_bytes, per_head = algorithmic_bytes(w, args.fit_every)
     peak, peak_kind = peaks()
@@ -332,7 +365,7 @@ def main():
     # the previous chunk, and readouts stream back (qstate_scan_host).
     e2e = None
     if not args.no_e2e:
-        names = ["q", "k", "v", "s", "beta"]
+        names = ["q", "k", "v", "s"] + (["beta"] if w.erase else [])
         host_in = {n: torch.empty(x[n].shape, dtype=x[n].dtype, pin_memory=True) for n in names}
         for n in names:
             host_in[n].copy_(x[n])
@@ -341,13 +374,15 @@ def main():
         d2h = host_o.numel() * host_o.element_size()
         comp, copy_stream = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
         comp.wait_stream(stream)
-        xh = q.Inputs(host_in["q"], host_in["k"], host_in["v"], None, None, None, host_in["beta"], w.T)
-        chunk = 64
+        xh = q.Inputs(host_in["q"], host_in["k"], host_in["v"], None if coded else host_in["s"],
+                      None, None, host_in.get("beta"), w.T)
+        chunk = max(64, w.C)
 
         def e2e_step():
-            with torch.cuda.stream(comp):
-                x["s"].copy_(host_in["s"], non_blocking=True)
-            q.qstate_quant_decay(cfg, x["s"], codes, lut, thr, comp)
+            if coded:   # the levels are taken over all tokens: the rates go first
+                with torch.cuda.stream(comp):
+                    x["s"].copy_(host_in["s"], non_blocking=True)
+                quant_decay(comp)
             q.qstate_init(cfg, A, Bst, comp)
             q.qstate_scan_host(cfg, A, Bst, xh, X, 0, w.T, 0, host_o, o, st, chunk, comp,
                                copy_stream)
@@ -370,7 +405,7 @@ def main():
 
     # decay quantiser (4), init (alloc + pack), then per write-back: write-back + alloc, or with
     # current-statistics allocation a statistics pass + alloc + write-back
-    launches_per_step = 4 + 2 + (3 if args.alloc_mode == 1 else 2) * w.T
+    launches_per_step = (4 if coded else 0) + 2 + (3 if args.alloc_mode == 1 else 2) * n_wb
     clocks = clk.summary()
     if rank != 0:
         if world > 1:
