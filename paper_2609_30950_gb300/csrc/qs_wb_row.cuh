@@ -27,8 +27,10 @@
 //       decay folded in, erase vector, k.q         -> unpack into registers (update layout),
 //       partials p = a^T S', r = q^T S'
 //   B3  -> u = beta v - p, o = r + u (k.q)
-//   B4  -> S = S' + k u^T (further tokens of the interval repeat B3..B4); the next head's
-//       packed rows are copied; state to the buffer
+//   B4  -> S = S' + k u^T.  Further tokens of the interval repeat from the partials, with
+//       their inputs prepared one token ahead in a second buffer (prefetched into L1 one more
+//       token ahead), so each token costs two barriers.  Then the next head's packed rows are
+//       copied and the state goes to the buffer
 //   B5  -> write-back (row layout): row range R, the 16 candidate steps and their squared
 //       errors (refit), codes, and each lane's packed words stored to the output region
 //   B6  -> coalesced stores of scales, factor indices, ranges and EMAs.
@@ -79,13 +81,19 @@ struct alignas(16) WbSmem {
     } rc;
     float4 deq[DK];                       // (-A, S, B, 0): x = (2^23 + u - A) S + B
     float4 wc[17];                        // per width: (n, 1/n, 2^23*1.5 - n, 2^23*1.5 + n)
-    float tk[DK], tq[DK], tv[DV];         // inputs of tokens after the first (C > 1)
-    float tw[DV];                         // general erasure: w of tokens after the first
-    float a[DK], d[DK];                   // erase vector beta k, decay of the current token
+    // token inputs, double-buffered by token parity (C > 1; k triple-buffered by token index
+    // mod 3).  Buffer 0 of the head's first token is the stage (k, q, v, w) with a and d here;
+    // later tokens alternate between buffer 1 (tk, tq, tv, tw, a1, d1) and buffer 0 (the
+    // stage's arrays, a, d); k takes the stage, tk and tk2 in turn.
+    float tk[DK], tk2[DK], tq[DK], tv[DV];
+    float tw[DV];                         // general erasure: w
+    float a[DK], d[DK];                   // erase vector a (beta k), decay (buffer 0)
+    float a1[DK], d1[DK];                 // (buffer 1)
+    float tbeta[2];
     float u[DV];
     float rowR[DK];
     float fitf[kNFit];
-    float wsum[NW];
+    float wsum[2][NW];                    // k.q partials per warp of rows, by buffer
     alignas(16) int off_in[DK + 4];
     alignas(16) int off_out[DK + 4];
     int cnt[1][17];
@@ -117,6 +125,9 @@ __device__ __forceinline__ void cp_async8(void* smem, const void* gmem) {
 __device__ __forceinline__ void cp_async4(void* smem, const void* gmem) {
     const unsigned s = static_cast<unsigned>(__cvta_generic_to_shared(smem));
     asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(s), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void prefetch_l1(const void* gmem) {
+    asm volatile("prefetch.global.L1 [%0];\n" ::"l"(gmem));
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
@@ -493,7 +504,7 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
             sm.a[i] = ai;
             // k . q: one partial per warp of rows
             const float kq = warp_sum(kk * S.q[i]);
-            if (lane == 0) sm.wsum[(tid - 64) >> 5] = kq;
+            if (lane == 0) sm.wsum[0][(tid - 64) >> 5] = kq;
         } else if (warp == 6) {
             // rows in order of output width (counting sort; any order within a width)
             const uint8_t* wa = S.w_out;
@@ -554,67 +565,100 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
         }
 
         // ---- tokens of the interval (Eq. 1) ----------------------------------------------------
-        for (int t = p.t_begin; t < p.t_end; ++t) {
+        // Per token: (A) the last DK threads first prepare the next token's inputs (decay, a,
+        // statistics, k.q) in the other buffer, loading them from L1 where they were prefetched
+        // one token earlier; then every warp applies the decay (tokens after the first; the
+        // first one's is folded into the dequantisation) and forms the partials p = S'^T a,
+        // r = S'^T q; B3; (B) the first DV threads take the column sums, u = w o v - p and
+        // o = r + u (k.q), while the input threads prefetch the token after next; B4;
+        // (C) S = S' + k u^T.
+        constexpr int P0 = NW * 32 - DK;   // first thread of the input-preparing role
+        static_assert(P0 >= DV, "the two roles of the middle phase overlap");
+        const int pi = tid - P0;
+        const bool prep_k = pi >= 0, prep_v = pi >= 0 && pi < DV;
+        // Token inputs are pulled into L1 one token ahead of their loads (prefetches hold no
+        // registers; the loads then hit L1).  The per-token stride of every input is H rows.
+        auto prefetch = [&](const float* kp, const float* qp, const void* sp, const float* bp,
+                            const float* vp) {
+            prefetch_l1(kp);
+            prefetch_l1(qp);
+            if (p.decay_row || pi == 0) prefetch_l1(sp);
+            if (p.erase && pi == 0) prefetch_l1(bp);
+            if (prep_v) prefetch_l1(vp);
+        };
+        if (prep_k && p.t_begin + 1 < p.t_end) {
+            const size_t tn = tok0 + p.H;
+            const size_t si = p.decay_row ? tn * DK + pi : tn;
+            prefetch(p.k + tn * DK + pi, p.q + tn * DK + pi,
+                     p.s_code ? static_cast<const void*>(p.s_code + si) : static_cast<const void*>(p.s + si),
+                     p.beta + tn, p.v + tn * DV + pi);
+        }
+        for (int t = p.t_begin, j = 0; t < p.t_end; ++t, ++j) {
             const size_t tok = (static_cast<size_t>(b) * T + t) * p.H + h;
-            const float* kv = S.k;
-            const float* qv = S.q;
-            const float* vv = S.v;
-            float beta = beta0;
-            float kq;
-            if (t > p.t_begin) {
-                __syncthreads();   // every warp is done with the previous token's k and u
-                beta = p.erase ? __ldg(p.beta + tok) : 1.0f;
-                float rh = 0.0f;
-                if (!p.decay_row)
-                    rh = p.s_code ? __ldg(p.s_lut + static_cast<size_t>(h) * p.L +
-                                          min(static_cast<int>(p.s_code[tok]), p.L - 1))
-                                  : __ldg(p.s + tok);
-                if (tid < DK) {
-                    const int i = tid;
-                    const float kk = __ldg(p.k + tok * DK + i), qq = __ldg(p.q + tok * DK + i);
-                    sm.tk[i] = kk;
-                    sm.tq[i] = qq;
-                    float rate = rh;
+            const int cb = j & 1, k3 = j % 3;
+            if (prep_k && t + 1 < p.t_end) {
+                // the next token's inputs into buffer cb ^ 1, whose contents (the previous
+                // token's) were last read before the previous B4.  k goes to the third k
+                // buffer: the previous token's k is read after that B4, the one before it was
+                // last read before the previous B3.
+                const int i = pi, nb = cb ^ 1, nk3 = k3 == 2 ? 0 : k3 + 1;
+                const size_t tn = tok + p.H;   // token t + 1 of this head
+                const float* kp = p.k + tn * DK + i;
+                const float* qp = p.q + tn * DK + i;
+                const float* vp = p.v + tn * DV + i;
+                const float* bp = p.beta + tn;
+                const size_t si = p.decay_row ? tn * DK + i : tn;
+                const float nbeta = p.erase ? __ldg(bp) : 1.0f;
+                const float nk = __ldg(kp), nq = __ldg(qp);
+                float rate;
+                if (p.s_code) {
+                    const int code = min(static_cast<int>(p.s_code[si]), p.L - 1);
                     if (p.decay_row)
-                        rate = p.s_code ? __ldg(p.s_lut + (static_cast<size_t>(h) * DK + i) * p.L +
-                                                min(static_cast<int>(p.s_code[tok * DK + i]), p.L - 1))
-                                        : __ldg(p.s + tok * DK + i);
-                    if (!(rate > 0.0f) || !(rate < INFINITY)) raise_status(p.status, QS_DEV_RATE);
-                    sm.d[i] = expf(-rate);
-                    sm.a[i] = p.general ? __ldg(p.a_in + tok * DK + i) : __fmul_rn(beta, kk);
-                    if (stats) {
-                        const float xs = -expm1f(-2.0f * rate);
-                        if (p.general) {
-                            sm.rowR[i] = xs;   // the erasure term needs all of k: after the barrier
-                        } else {
-                            const float xr = p.erase ? __fmul_rn(__fmul_rn(beta, __fsub_rn(2.0f, beta)), __fmul_rn(kk, kk)) : 0.0f;
-                            S.ms[i] = __fadd_rn(S.ms[i], __fmul_rn(p.alpha, __fsub_rn(xs, S.ms[i])));
-                            S.mr[i] = __fadd_rn(S.mr[i], __fmul_rn(p.alpha, __fsub_rn(xr, S.mr[i])));
-                        }
+                        rate = p.L <= 4 ? S.lut[i * p.L + code]
+                                        : __ldg(p.s_lut + (static_cast<size_t>(h) * DK + i) * p.L + code);
+                    else
+                        rate = __ldg(p.s_lut + static_cast<size_t>(h) * p.L + code);
+                } else {
+                    rate = __ldg(p.s + si);
+                }
+                if (!(rate > 0.0f) || !(rate < INFINITY)) raise_status(p.status, QS_DEV_RATE);
+                (nk3 == 0 ? S.k : nk3 == 1 ? sm.tk : sm.tk2)[i] = nk;
+                (nb ? sm.tq : S.q)[i] = nq;
+                (nb ? sm.d1 : sm.d)[i] = expf(-rate);
+                (nb ? sm.a1 : sm.a)[i] = p.general ? __ldg(p.a_in + tn * DK + i) : __fmul_rn(nbeta, nk);
+                if (prep_v) {
+                    (nb ? sm.tv : S.v)[i] = __ldg(vp);
+                    if (p.general) (nb ? sm.tw : S.gw)[i] = __ldg(p.w_in + tn * DV + i);
+                }
+                if (i == 0) sm.tbeta[nb] = nbeta;
+                if (stats) {
+                    const float xs = -expm1f(-2.0f * rate);
+                    if (p.general) {
+                        sm.rowR[i] = xs;   // the erasure term needs all of the next k: after B3
+                    } else {
+                        const float xr = p.erase ? __fmul_rn(__fmul_rn(nbeta, __fsub_rn(2.0f, nbeta)), __fmul_rn(nk, nk)) : 0.0f;
+                        S.ms[i] = __fadd_rn(S.ms[i], __fmul_rn(p.alpha, __fsub_rn(xs, S.ms[i])));
+                        S.mr[i] = __fadd_rn(S.mr[i], __fmul_rn(p.alpha, __fsub_rn(xr, S.mr[i])));
                     }
-                    const float s2 = warp_sum(kk * qq);
-                    if (lane == 0) sm.wsum[warp] = s2;
                 }
-                if (tid < DV) {
-                    sm.tv[tid] = __ldg(p.v + tok * DV + tid);
-                    if (p.general) sm.tw[tid] = __ldg(p.w_in + tok * DV + tid);
-                }
-                __syncthreads();
-                if (p.general && stats && tid < DK) {
-                    const float xs = sm.rowR[tid];
-                    const float xr = general_erasure<DK>(sm.a[tid], sm.tk[tid], sm.tk);
-                    S.ms[tid] = __fadd_rn(S.ms[tid], __fmul_rn(p.alpha, __fsub_rn(xs, S.ms[tid])));
-                    S.mr[tid] = __fadd_rn(S.mr[tid], __fmul_rn(p.alpha, __fsub_rn(xr, S.mr[tid])));
-                }
-                kv = sm.tk;
-                qv = sm.tq;
-                vv = sm.tv;
+                const float s2 = warp_sum(nk * nq);
+                if (lane == 0) sm.wsum[nb][i >> 5] = s2;
+            }
+            const float* kv = k3 == 0 ? S.k : k3 == 1 ? sm.tk : sm.tk2;
+            const float* qv = cb ? sm.tq : S.q;
+            const float* av = cb ? sm.a1 : sm.a;
+            if (j > 0) {
+                const float* dd = cb ? sm.d1 : sm.d;
 #pragma unroll
-                for (int r = 0; r < RPW; ++r) {
-                    const float dd = sm.d[warp * RPW + r];
-                    const float2 d2 = make_float2(dd, dd);
+                for (int r4 = 0; r4 < RPW; r4 += 4) {
+                    const float4 d4 = *reinterpret_cast<const float4*>(&dd[warp * RPW + r4]);
+                    const float ds[4] = {d4.x, d4.y, d4.z, d4.w};
 #pragma unroll
-                    for (int c = 0; c < CP2; ++c) x[r][c] = __fmul2_rn(x[r][c], d2);
+                    for (int j4 = 0; j4 < 4; ++j4) {
+                        const float2 d2 = make_float2(ds[j4], ds[j4]);
+#pragma unroll
+                        for (int c = 0; c < CP2; ++c) x[r4 + j4][c] = __fmul2_rn(x[r4 + j4][c], d2);
+                    }
                 }
             }
             float2 pp[CP2], rr[CP2];
@@ -622,7 +666,7 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
             for (int c = 0; c < CP2; ++c) pp[c] = rr[c] = make_float2(0.0f, 0.0f);
 #pragma unroll
             for (int r4 = 0; r4 < RPW; r4 += 4) {
-                const float4 a4 = *reinterpret_cast<const float4*>(&sm.a[warp * RPW + r4]);
+                const float4 a4 = *reinterpret_cast<const float4*>(&av[warp * RPW + r4]);
                 const float4 q4 = *reinterpret_cast<const float4*>(&qv[warp * RPW + r4]);
                 const float as[4] = {a4.x, a4.y, a4.z, a4.w}, qs[4] = {q4.x, q4.y, q4.z, q4.w};
 #pragma unroll
@@ -649,15 +693,32 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                     P += sm.rc.red[0][w][jv];
                     Rr += sm.rc.red[1][w][jv];
                 }
-                kq = 0.0f;
+                float kq = 0.0f;
 #pragma unroll
-                for (int w = 0; w < DK / 32; ++w) kq += sm.wsum[w];
-                const float vj = vv[jv];
+                for (int w = 0; w < DK / 32; ++w) kq += sm.wsum[cb][w];
+                const float vj = (cb ? sm.tv : S.v)[jv];
+                const float beta = j == 0 ? beta0 : sm.tbeta[cb];
                 // u = w o v - p (w = beta 1 for the delta rule; a = 0, w = 1 without erasure)
-                const float wj = p.general ? (t > p.t_begin ? sm.tw[jv] : S.gw[jv]) : beta;
+                const float wj = p.general ? (cb ? sm.tw : S.gw)[jv] : beta;
                 const float uu = (p.erase || p.general) ? __fsub_rn(__fmul_rn(wj, vj), P) : vj;
                 sm.u[jv] = uu;
                 p.o[tok * DV + jv] = fmaf(uu, kq, Rr);
+            } else if (prep_k && t + 1 < p.t_end) {
+                if (t + 2 < p.t_end) {   // the token after next, into L1
+                    const size_t tn = tok + 2 * static_cast<size_t>(p.H);
+                    const size_t si = p.decay_row ? tn * DK + pi : tn;
+                    prefetch(p.k + tn * DK + pi, p.q + tn * DK + pi,
+                             p.s_code ? static_cast<const void*>(p.s_code + si) : static_cast<const void*>(p.s + si),
+                             p.beta + tn, p.v + tn * DV + pi);
+                }
+                if (p.general && stats) {
+                    // the general erasure statistic of the next token (needs all of its k)
+                    const int nk3 = k3 == 2 ? 0 : k3 + 1;
+                    const float* kb = nk3 == 0 ? S.k : nk3 == 1 ? sm.tk : sm.tk2;
+                    const float xr = general_erasure<DK>((cb ? sm.a : sm.a1)[pi], kb[pi], kb);
+                    S.ms[pi] = __fadd_rn(S.ms[pi], __fmul_rn(p.alpha, __fsub_rn(sm.rowR[pi], S.ms[pi])));
+                    S.mr[pi] = __fadd_rn(S.mr[pi], __fmul_rn(p.alpha, __fsub_rn(xr, S.mr[pi])));
+                }
             }
             __syncthreads();                                                           // B4
             float2 u2[CP2];

@@ -405,6 +405,29 @@ def test_quantised_lockstep_weight_kinds(qs, orc, kind):
     _lockstep(qs, orc, SMALL["kda_decode"], log_decay=True, weight_kind=kind)
 
 
+CHUNKED_ROW_CASES = {
+    "coded_g2": (lambda: small("kda_decode", B=2, H=3, T=19, C=8), True),
+    "coded_g3": (lambda: small("kda_decode", B=2, H=3, T=13, C=5, gate_bits=3), True),
+    "mamba2": (lambda: small("mamba2_decode", B=2, H=16, T=17, C=8), False),
+    "tiny": (lambda: small("tiny_kda", T=23, C=7), False),
+    "general": (lambda: synth.scaled(synth.EXTENSION_WORKLOADS["kda_general"], B=2, H=3, T=20, C=6), False),
+    "persistent": (lambda: synth.scaled(synth.EXTENSION_WORKLOADS["kda_persistent"], B=2, H=3, T=14, C=4), True),
+}
+
+
+@pytest.mark.parametrize("case", sorted(CHUNKED_ROW_CASES))
+def test_quantised_lockstep_chunked_row_kernel(qs, orc, case):
+    """Write-back periods C > 1 through the row-unit kernel, whose tokens after the first take
+    their inputs from alternating buffers filled one token ahead: log-coded rates from the
+    head's level table (g = 2) and from the global table (g = 3), per-head rates without
+    erasure (Mamba-2, dv = 64), 64 x 64 heads, general a and w, persistent decay; every case
+    ends on a ragged interval."""
+    make, log_decay = CHUNKED_ROW_CASES[case]
+    w = make()
+    assert w.C > 1 and w.T % w.C != 0
+    _lockstep(qs, orc, w, log_decay=log_decay)
+
+
 def test_quantised_lockstep_ragged_chunks(qs, orc):
     w = small("kda_prefill", B=1, H=2, T=37, C=16)
     _lockstep(qs, orc, w)
