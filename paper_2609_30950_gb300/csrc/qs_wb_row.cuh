@@ -17,22 +17,24 @@
 //    l CPL w of the row, for any width w).
 //  * row layout: TPR = dv/32 lanes per row, each owning 32 consecutive value columns, i.e. a
 //    word-aligned run of 32 codes (4w bytes).  Warps take rows in order of output width (a
-//    counting sort per head), so the code arithmetic of a warp is specialised for one width.
+//    sort per head), so the code arithmetic of a warp is specialised for one width.
 //    Used for the write-back (range, factor search, codes, packing); the state reaches it
 //    through a shared-memory buffer (16-byte groups XOR-swizzled per row).
 // Per head there are six CTA barriers:
-//   B1  the head's inputs have landed            -> issue the next head's metadata copies
-//   B2  prep: row offsets (prefix sums of widths), rows sorted by output width, layout
-//       checks, per-row decay, EMA update, dequantisation constants with the first token's
-//       decay folded in, erase vector, k.q         -> unpack into registers (update layout),
+//   B1  the head's inputs have landed            -> prep, one role per warp group: row offsets
+//       (prefix sums of widths) and layout checks; per-row decay, EMA update, dequantisation
+//       constants with the first token's decay folded in, erase vector, k.q; rows sorted by
+//       output width; and, on the last warp, the next head's metadata copies
+//   B2  -> unpack into registers (update layout),
 //       partials p = a^T S', r = q^T S'
 //   B3  -> u = beta v - p, o = r + u (k.q)
 //   B4  -> S = S' + k u^T.  Further tokens of the interval repeat from the partials, with
 //       their inputs prepared one token ahead in a second buffer (prefetched into L1 one more
 //       token ahead), so each token costs two barriers.  Then the next head's packed rows are
 //       copied and the state goes to the buffer
-//   B5  -> write-back (row layout): row range R, the 16 candidate steps and their squared
-//       errors (refit), codes, and each lane's packed words stored to the output region
+//   B5  -> write-back (row layout), batches of rows claimed dynamically: row range R, the 16
+//       candidate steps and their squared errors (refit), codes, and each lane's packed
+//       words stored to the output region
 //   B6  -> coalesced stores of scales, factor indices, ranges and EMAs.
 // The next head's B1 orders the reuse of stage and staging buffers.
 #pragma once
@@ -96,11 +98,11 @@ struct alignas(16) WbSmem {
     float wsum[2][NW];                    // k.q partials per warp of rows, by buffer
     alignas(16) int off_in[DK + 4];
     alignas(16) int off_out[DK + 4];
-    int cnt[1][17];
     uint8_t ord_out[DK];                  // rows in order of output width
     uint16_t out_scale[DK];
     uint8_t out_fidx[DK];
     int flag;
+    int bat_next;                         // next row batch of the write-back to claim
 };
 
 // Float offset of 16-byte group G of row i in the state buffer.  The XOR keeps each group in
@@ -275,66 +277,53 @@ __device__ __forceinline__ void pack_row(int w, const float2 (&xv)[16], float in
     }
 }
 
-// Issue the asynchronous copies of head g's metadata into stage S.  The head's payload window
-// (in_off, in_end) and output offset come from the previous stage (or, for the first head, from
-// direct loads) and are checked here; gnext >= 0 names the head whose offsets to fetch.  One
-// commit group per call.
+// Issue the asynchronous copies of head g's metadata into stage S, by threads t = 0..nt-1 of
+// the calling group (the whole CTA for a CTA's first head; one warp, which has no other work in
+// the prep phase, for the heads after it).  The head's payload window (in_off, in_end) and output
+// offset come from the previous stage (or, for the first head, from direct loads) and are checked
+// here; gnext >= 0 names the head whose offsets to fetch.  One commit group per call.
 template <int DK, int DV>
-__device__ __noinline__ void wb_issue_meta(WbStage<DK, DV>& S, int g, int gnext, int in_off, int in_end,
-                                           int out_off, const WbParams& wp) {
+__device__ __forceinline__ void wb_issue_meta(WbStage<DK, DV>& S, int g, int gnext, int in_off, int in_end,
+                                           int out_off, const WbParams& wp, int t, int nt) {
     const StepParams& p = wp.s;
-    const int tid = threadIdx.x;
     const bool stats = p.ema_s != nullptr;
     const int T = p.T;
     const int b = g / p.H, h = g - (g / p.H) * p.H;
     const size_t tok = (static_cast<size_t>(b) * T + p.t_begin) * p.H + h;
     const size_t rb = static_cast<size_t>(g) * DK;
-    // fixed-size arrays, 16-byte chunks
+    // one array at a time, in 16-byte chunks
+    auto seg = [&](void* dst, const void* src, int nchunks) {
+        for (int c = t; c < nchunks; c += nt)
+            cp_async16(static_cast<uint8_t*>(dst) + 16 * c, static_cast<const uint8_t*>(src) + 16 * c);
+    };
     constexpr int C8 = DK / 16, C16 = DK * 2 / 16, C32 = DK * 4 / 16, CV = DV * 4 / 16;
-    int c = tid;
-    if (c < C8) cp_async16(S.w_in + 16 * c, p.in_widths + rb + 16 * c);
-    else if ((c -= C8) < C8) cp_async16(S.w_out + 16 * c, p.out_widths + rb + 16 * c);
-    else if ((c -= C8) < C8) cp_async16(S.fidx + 16 * c, p.in_fidx + rb + 16 * c);
-    else if ((c -= C8) < C16) cp_async16(reinterpret_cast<uint8_t*>(S.sc_in) + 16 * c,
-                                         reinterpret_cast<const uint8_t*>(p.in_scales + rb) + 16 * c);
-    else if ((c -= C16) < C32) cp_async16(reinterpret_cast<uint8_t*>(S.k) + 16 * c,
-                                          reinterpret_cast<const uint8_t*>(p.k + tok * DK) + 16 * c);
-    else if ((c -= C32) < C32) cp_async16(reinterpret_cast<uint8_t*>(S.q) + 16 * c,
-                                          reinterpret_cast<const uint8_t*>(p.q + tok * DK) + 16 * c);
-    else if ((c -= C32) < CV) cp_async16(reinterpret_cast<uint8_t*>(S.v) + 16 * c,
-                                         reinterpret_cast<const uint8_t*>(p.v + tok * DV) + 16 * c);
-    else if ((c -= CV) < C32) {
-        if (stats) cp_async16(reinterpret_cast<uint8_t*>(S.ms) + 16 * c,
-                              reinterpret_cast<const uint8_t*>(p.ema_s + rb) + 16 * c);
-    } else if ((c -= C32) < C32) {
-        if (stats) cp_async16(reinterpret_cast<uint8_t*>(S.mr) + 16 * c,
-                              reinterpret_cast<const uint8_t*>(p.ema_r + rb) + 16 * c);
-    } else if ((c -= C32) < C32) {
-        if (p.decay_row && !p.s_code) cp_async16(reinterpret_cast<uint8_t*>(S.s) + 16 * c,
-                                                 reinterpret_cast<const uint8_t*>(p.s + tok * DK) + 16 * c);
-    } else if ((c -= C32) < C8) {
-        if (p.decay_row && p.s_code) cp_async16(S.scode + 16 * c, p.s_code + tok * DK + 16 * c);
+    seg(S.w_in, p.in_widths + rb, C8);
+    seg(S.w_out, p.out_widths + rb, C8);
+    seg(S.fidx, p.in_fidx + rb, C8);
+    seg(S.sc_in, p.in_scales + rb, C16);
+    seg(S.k, p.k + tok * DK, C32);
+    seg(S.q, p.q + tok * DK, C32);
+    seg(S.v, p.v + tok * DV, CV);
+    if (stats) {
+        seg(S.ms, p.ema_s + rb, C32);
+        seg(S.mr, p.ema_r + rb, C32);
     }
+    if (p.decay_row && !p.s_code) seg(S.s, p.s + tok * DK, C32);
+    if (p.decay_row && p.s_code) seg(S.scode, p.s_code + tok * DK, C8);
     // general erasure: the first token's a (DK floats) and w (DV floats)
     if (p.general) {
-        for (int i = tid; i < DK / 4 + DV / 4; i += blockDim.x) {
-            if (i < DK / 4) cp_async16(S.ga + 4 * i, p.a_in + tok * DK + 4 * i);
-            else cp_async16(S.gw + 4 * (i - DK / 4), p.w_in + tok * DV + 4 * (i - DK / 4));
-        }
+        seg(S.ga, p.a_in + tok * DK, DK / 4);
+        seg(S.gw, p.w_in + tok * DV, DV / 4);
     }
-    // the head's decay levels (DK x L floats, 16-byte chunks) when L <= 4
-    if (p.decay_row && p.s_code && p.L <= 4) {
-        const int nch = DK * p.L / 4;
-        const float* src = p.s_lut + static_cast<size_t>(h) * DK * p.L;
-        for (int i = tid; i < nch; i += blockDim.x) cp_async16(S.lut + 4 * i, src + 4 * i);
-    }
+    // the head's decay levels (DK x L floats) when L <= 4
+    if (p.decay_row && p.s_code && p.L <= 4) seg(S.lut, p.s_lut + static_cast<size_t>(h) * DK * p.L, DK * p.L / 4);
     // scalars and the offsets of the next head
-    if (tid == blockDim.x - 1) {
+    if (t == nt - 1) {
         if (p.erase) cp_async4(&S.beta, p.beta + tok);
         if (!p.decay_row && !p.s_code) cp_async4(&S.rate_h, p.s + tok);
     }
     const bool next_last = gnext >= 0 && gnext - (gnext / p.H) * p.H == p.H - 1;
-    if (tid == blockDim.x - 2 && gnext >= 0) {
+    if (t == nt - 2 && gnext >= 0) {
         cp_async4(&S.nxt_in_off, p.in_head_off + gnext);
         cp_async4(&S.nxt_out_off, p.out_head_off + gnext);
         if (!next_last) cp_async4(&S.nxt_in_end, p.in_head_off + gnext + 1);
@@ -344,7 +333,7 @@ __device__ __noinline__ void wb_issue_meta(WbStage<DK, DV>& S, int g, int gnext,
     const int nbytes = in_end - in_off;
     const bool ok = in_off >= 0 && nbytes >= 0 && nbytes <= p.stage_bytes && in_off % align == 0 &&
                     nbytes % align == 0 && static_cast<long long>(in_end) <= p.region_bytes;
-    if (tid == 0) {
+    if (t == 0) {
         S.in_off = in_off;
         S.in_end = in_end;
         S.out_off = out_off;
@@ -359,7 +348,7 @@ __device__ __noinline__ void wb_issue_meta(WbStage<DK, DV>& S, int g, int gnext,
 // Copy head g's packed rows (the window recorded in S by wb_issue_meta; S.ok must be visible
 // to every thread) into pay.  One commit group per call.
 template <int DK, int DV>
-__device__ __noinline__ void wb_issue_payload(const WbStage<DK, DV>& S, uint8_t* pay, int g, const WbParams& wp) {
+__device__ __forceinline__ void wb_issue_payload(const WbStage<DK, DV>& S, uint8_t* pay, int g, const WbParams& wp) {
     const StepParams& p = wp.s;
     const int tid = threadIdx.x;
     if (S.ok) {
@@ -409,7 +398,8 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
         const int io = static_cast<int>(p.in_head_off[g_begin]);
         const int ie = h0 < p.H - 1 ? static_cast<int>(p.in_head_off[g_begin + 1]) : static_cast<int>(p.region_bytes);
         const int oo = static_cast<int>(p.out_head_off[g_begin]);
-        wb_issue_meta<DK, DV>(sm.st[0], g_begin, g_begin + 1 < g_end ? g_begin + 1 : -1, io, ie, oo, wp);
+        wb_issue_meta<DK, DV>(sm.st[0], g_begin, g_begin + 1 < g_end ? g_begin + 1 : -1, io, ie, oo, wp,
+                              tid, NW * 32);
         __syncthreads();
         wb_issue_payload<DK, DV>(sm.st[0], pay, g_begin, wp);
     }
@@ -422,9 +412,10 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
         if (tid == 0) sm.flag = S.ok ? 0 : 1;
         __syncthreads();                                                               // B1
         const bool has_next = g + 1 < g_end;
-        if (has_next)
+        // the next head's metadata, by the warp that has no prep role
+        if (has_next && warp == NW - 1)
             wb_issue_meta<DK, DV>(sm.st[sidx ^ 1], g + 1, g + 2 < g_end ? g + 2 : -1, S.nxt_in_off,
-                                  S.nxt_in_end, S.nxt_out_off, wp);
+                                  S.nxt_in_end, S.nxt_out_off, wp, lane, 32);
 
         // ---- prep ---------------------------------------------------------------------------
         const size_t tok0 = (static_cast<size_t>(b) * T + p.t_begin) * p.H + h;
@@ -506,32 +497,35 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
             const float kq = warp_sum(kk * S.q[i]);
             if (lane == 0) sm.wsum[0][(tid - 64) >> 5] = kq;
         } else if (warp == 6) {
-            // rows in order of output width (counting sort; any order within a width)
-            const uint8_t* wa = S.w_out;
-            uint8_t* ord = sm.ord_out;
-            int* cnt = sm.cnt[0];
-            if (lane < 17) cnt[lane] = 0;
-            __syncwarp();
+            // Rows in order of output width, any order within a width.  Widths 2..16 come
+            // first in ascending order (the narrowest rows have the longest range-factor
+            // search), then widths 1 and 0, so that the write-back's batches are claimed
+            // longest first.  A ballot per width present and slot gives every row its place.
             constexpr int PER = DK / 32;
-            int slot[PER], wv[PER];
+            int key[PER], pos[PER];
+            unsigned present = 0u;
 #pragma unroll
             for (int jj = 0; jj < PER; ++jj) {
-                wv[jj] = min(static_cast<int>(wa[lane * PER + jj]), 16);
-                slot[jj] = atomicAdd(&cnt[wv[jj]], 1);
+                key[jj] = (min(static_cast<int>(S.w_out[lane * PER + jj]), 16) + 15) % 17;
+                pos[jj] = 0;
+                present |= 1u << key[jj];
             }
-            __syncwarp();
-            const int c = lane < 17 ? cnt[lane] : 0;
-            int incl = c;
+            present = __reduce_or_sync(kFull, present);
+            const unsigned lt = (1u << lane) - 1u;
+            int base = 0;
+            while (present != 0u) {
+                const int kb = __ffs(present) - 1;
+                present &= present - 1u;
 #pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const int n = __shfl_up_sync(kFull, incl, o);
-                if (lane >= o) incl += n;
+                for (int jj = 0; jj < PER; ++jj) {
+                    const unsigned m = __ballot_sync(kFull, key[jj] == kb);
+                    if (key[jj] == kb) pos[jj] = base + __popc(m & lt);
+                    base += __popc(m);
+                }
             }
-            __syncwarp();
-            if (lane < 17) cnt[lane] = incl - c;
-            __syncwarp();
 #pragma unroll
-            for (int jj = 0; jj < PER; ++jj) ord[cnt[wv[jj]] + slot[jj]] = static_cast<uint8_t>(lane * PER + jj);
+            for (int jj = 0; jj < PER; ++jj) sm.ord_out[pos[jj]] = static_cast<uint8_t>(lane * PER + jj);
+            if (lane == 0) sm.bat_next = NW;
         }
         __syncthreads();                                                               // B2
         if (sm.flag != 0) {
@@ -753,7 +747,14 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
 
         // ---- write-back (row layout) ----------------------------------------------------------
         const bool refit = (p.fit_every <= 1) || ((p.w_index + h) % p.fit_every == 0);
-        for (int bat = warp; bat < NB; bat += NW) {
+        // Row batches are claimed dynamically (longest first, by the order above): the
+        // search length varies with the width and the data.
+        auto next_batch = [&]() {
+            int nb = 0;
+            if (lane == 0) nb = atomicAdd(&sm.bat_next, 1);
+            return __shfl_sync(kFull, nb, 0);
+        };
+        for (int bat = warp; bat < NB; bat = next_batch()) {
             const int i = sm.ord_out[bat * RPB + lane / TPR], q = lane % TPR;
             const int w = S.w_out[i];
             float2 xv[16], av[16];
@@ -805,10 +806,12 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                 __syncwarp();
                 // squared error of the candidates (levels clamped at n): e = |x| - q Delta,
                 // q = min(rint(|x| / Delta), n); the smallest wins, ties to the larger factor.
-                // Candidates are taken from the largest factor down.  Every element at or above
-                // n Delta_k quantises to n, so the clipping error of the lanes' maxima is a lower
-                // bound on candidate k's error that grows as k falls: once it exceeds the best
-                // error found (with a 2^-10 margin for rounding), no smaller factor can win.
+                // Candidates are taken from the largest factor down, two per round (independent
+                // work for the warp).  Every element at or above n Delta_k quantises to n, so the
+                // clipping error of the lanes' maxima is a lower bound on candidate k's error that
+                // grows as k falls: once it exceeds the best error found (with a 2^-10 margin for
+                // rounding), no smaller factor can win.  The round's second candidate is evaluated
+                // even when its bound already rules it out; it then cannot win the comparison.
                 const float lim = sm.wc[w > 16 ? 0 : w].w, nf = sm.wc[w > 16 ? 0 : w].x;
                 float mx[TPR];
 #pragma unroll
@@ -818,38 +821,55 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                 float bsse = INFINITY;
                 int bk = kNFit - 1;
 #pragma unroll 1
-                for (int k = kNFit - 1; k >= 0; --k) {
-                    const float2 cd = crow[k];
-                    const float Lk = -nf * cd.y;
-                    float lb = 0.0f;
+                for (int k = kNFit - 1; k >= 0; k -= 2) {
+                    // candidates k and k - 1 in one round (k - 1 may not exist)
+                    const bool two = k >= 1;
+                    const float2 cA = crow[k], cB = crow[two ? k - 1 : k];
+                    const float LA = -nf * cA.y, LB = -nf * cB.y;
+                    float lbA = 0.0f;
 #pragma unroll
                     for (int jl = 0; jl < TPR; ++jl) {
-                        const float e = fmaxf(mx[jl] - Lk, 0.0f);
-                        lb = fmaf(e, e, lb);
+                        const float e = fmaxf(mx[jl] - LA, 0.0f);
+                        lbA = fmaf(e, e, lbA);
                     }
-                    const bool go = w >= 2 && lb <= bsse * (1.0f + 1.0f / 1024.0f);
-                    if (!__any_sync(kFull, go)) break;
-                    const float2 i2 = make_float2(cd.x, cd.x), d2 = make_float2(cd.y, cd.y);
-                    float2 acc0 = make_float2(0.0f, 0.0f), acc1 = make_float2(0.0f, 0.0f);
+                    const bool goA = w >= 2 && lbA <= bsse * (1.0f + 1.0f / 1024.0f);
+                    if (!__any_sync(kFull, goA)) break;
+                    const float2 iA = make_float2(cA.x, cA.x), dA = make_float2(cA.y, cA.y);
+                    const float2 iB = make_float2(cB.x, cB.x), dB = make_float2(cB.y, cB.y);
+                    float2 aA0 = make_float2(0.0f, 0.0f), aA1 = aA0, aB0 = aA0, aB1 = aA0;
 #pragma unroll
                     for (int c = 0; c < 16; c += 2) {
-                        float2 t0 = __ffma2_rn(av[c], i2, M2);
-                        float2 t1 = __ffma2_rn(av[c + 1], i2, M2);
-                        t0.x = fminf(t0.x, lim);
-                        t0.y = fminf(t0.y, lim);
-                        t1.x = fminf(t1.x, lim);
-                        t1.y = fminf(t1.y, lim);
-                        const float2 e0 = __ffma2_rn(__fadd2_rn(t0, nM2), d2, av[c]);
-                        const float2 e1 = __ffma2_rn(__fadd2_rn(t1, nM2), d2, av[c + 1]);
-                        acc0 = __ffma2_rn(e0, e0, acc0);
-                        acc1 = __ffma2_rn(e1, e1, acc1);
+                        float2 t0 = __ffma2_rn(av[c], iA, M2);
+                        float2 t1 = __ffma2_rn(av[c + 1], iA, M2);
+                        float2 u0 = __ffma2_rn(av[c], iB, M2);
+                        float2 u1 = __ffma2_rn(av[c + 1], iB, M2);
+                        t0.x = fminf(t0.x, lim); t0.y = fminf(t0.y, lim);
+                        t1.x = fminf(t1.x, lim); t1.y = fminf(t1.y, lim);
+                        u0.x = fminf(u0.x, lim); u0.y = fminf(u0.y, lim);
+                        u1.x = fminf(u1.x, lim); u1.y = fminf(u1.y, lim);
+                        const float2 e0 = __ffma2_rn(__fadd2_rn(t0, nM2), dA, av[c]);
+                        const float2 e1 = __ffma2_rn(__fadd2_rn(t1, nM2), dA, av[c + 1]);
+                        const float2 f0 = __ffma2_rn(__fadd2_rn(u0, nM2), dB, av[c]);
+                        const float2 f1 = __ffma2_rn(__fadd2_rn(u1, nM2), dB, av[c + 1]);
+                        aA0 = __ffma2_rn(e0, e0, aA0);
+                        aA1 = __ffma2_rn(e1, e1, aA1);
+                        aB0 = __ffma2_rn(f0, f0, aB0);
+                        aB1 = __ffma2_rn(f1, f1, aB1);
                     }
-                    float tot = (acc0.x + acc0.y) + (acc1.x + acc1.y);
+                    float tA = (aA0.x + aA0.y) + (aA1.x + aA1.y);
+                    float tB = (aB0.x + aB0.y) + (aB1.x + aB1.y);
 #pragma unroll
-                    for (int o = 1; o < TPR; o <<= 1) tot += __shfl_xor_sync(kFull, tot, o);
-                    if (go && tot < bsse) {
-                        bsse = tot;
+                    for (int o = 1; o < TPR; o <<= 1) {
+                        tA += __shfl_xor_sync(kFull, tA, o);
+                        tB += __shfl_xor_sync(kFull, tB, o);
+                    }
+                    if (goA && tA < bsse) {
+                        bsse = tA;
                         bk = k;
+                    }
+                    if (two && w >= 2 && tB < bsse) {
+                        bsse = tB;
+                        bk = k - 1;
                     }
                 }
                 if (w >= 2) {
