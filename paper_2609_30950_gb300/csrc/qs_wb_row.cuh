@@ -81,7 +81,8 @@ struct alignas(16) WbSmem {
         float2 cand[NW][32 / (DV / 32)][kNFit + 1];   // per warp and row: (1/Delta_k, -Delta_k)
                                                       // (rows padded against bank conflicts)
     } rc;
-    float4 deq[DK];                       // (-A, S, B, 0): x = (2^23 + u - A) S + B
+    float4 deqAS[DK];                     // (-A, -A, S, S) and (B, B): x = (2^23 + u - A) S + B,
+    float2 deqB[DK];                      // as pairs, the operands of packed FP32 arithmetic
     float4 wc[17];                        // per width: (n, 1/n, 2^23*1.5 - n, 2^23*1.5 + n)
     // token inputs, double-buffered by token parity (C > 1; k triple-buffered by token index
     // mod 3).  Buffer 0 of the head's first token is the stage (k, q, v, w) with a and d here;
@@ -138,93 +139,29 @@ __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wai
 // The lane's codes occupy the 4W bytes at byte 4 W q of the row (q = its part), a whole number of
 // words: code c of the run sits at bits [c W, c W + W) of those words.
 
+// Packing.  With t_c = fl(x_c / Delta) + kMagic (round to nearest even; its bit pattern is
+// kMagicBits + q_c), the stored code u_c = clamp(q_c + n, 0, 2n) is one add-min-relu on the bits;
+// codes are shifted into the lane's words (codes that straddle two words add their high bits to
+// the next word).
 template <int W, int C>
-__device__ __forceinline__ uint32_t run_code(const uint32_t (&wd)[W + 1]) {
+__device__ __forceinline__ void run_put(uint32_t (&wd)[W], uint32_t u) {
     constexpr int bp = C * W, k = bp >> 5, sh = bp & 31;
-    constexpr uint32_t mask = (W >= 32) ? 0xffffffffu : ((1u << W) - 1u);
-    if constexpr (sh + W <= 32) return (wd[k] >> sh) & mask;
-    else return __funnelshift_r(wd[k], wd[k + 1], sh) & mask;
-}
-
-template <int W, int C>
-struct RunDecode {
-    __device__ __forceinline__ static void go(const uint32_t (&wd)[W + 1], float2 (&v)[16], float2 A2, float2 S2, float2 B2) {
-        const float2 t = make_float2(__uint_as_float(kTwo23Bits | run_code<W, C>(wd)),
-                                     __uint_as_float(kTwo23Bits | run_code<W, C + 1>(wd)));
-        v[C / 2] = __ffma2_rn(__fadd2_rn(t, A2), S2, B2);
-        RunDecode<W, C + 2>::go(wd, v, A2, S2, B2);
-    }
-};
-template <int W>
-struct RunDecode<W, 32> {
-    __device__ __forceinline__ static void go(const uint32_t (&)[W + 1], float2 (&)[16], float2, float2, float2) {}
-};
-
-// Unpack + dequantise the lane's 32 codes (row i, part q) into the state buffer.
-template <int W, int DV>
-__device__ __forceinline__ void unpack_run(const uint8_t* src, const float4 dq, float* sb, int i, int q) {
-    float2 v[16];
-    const float2 A2 = make_float2(dq.x, dq.x), S2 = make_float2(dq.y, dq.y), B2 = make_float2(dq.z, dq.z);
-    if constexpr (W == 0) {
-#pragma unroll
-        for (int k = 0; k < 16; ++k) v[k] = B2;
-    } else {
-        uint32_t wd[W + 1];
-#pragma unroll
-        for (int k = 0; k < W; ++k) wd[k] = reinterpret_cast<const uint32_t*>(src)[k];
-        wd[W] = 0u;
-        RunDecode<W, 0>::go(wd, v, A2, S2, B2);
-    }
-#pragma unroll
-    for (int g = 0; g < 8; ++g)
-        *reinterpret_cast<float4*>(sb + sb_off<DV>(i, 8 * q + g)) =
-            make_float4(v[2 * g].x, v[2 * g].y, v[2 * g + 1].x, v[2 * g + 1].y);
-}
-
-template <int DV>
-__device__ __forceinline__ void unpack_row(int w, const uint8_t* src, const float4 dq, float* sb, int i, int q) {
-    switch (w) {
-#define QS_W(N) case N: unpack_run<N, DV>(src, dq, sb, i, q); break;
-        QS_W(0) QS_W(1) QS_W(2) QS_W(3) QS_W(4) QS_W(5) QS_W(6) QS_W(7) QS_W(8)
-        QS_W(9) QS_W(10) QS_W(11) QS_W(12) QS_W(13) QS_W(14) QS_W(15) QS_W(16)
-#undef QS_W
-        default: break;
-    }
-}
-
-// Packing.  With b_c the bit pattern of kMagic + q_c (= kMagicBits + q_c), the stored code is
-// u_c = q_c + n = b_c + (n - kMagicBits) (mod 2^32), so each word is a sum of b_c << sh_c plus a
-// per-word constant: one integer multiply-add per code (codes that straddle two words add their
-// high bits to the next word separately).
-template <int W>
-__host__ __device__ constexpr uint32_t run_pack_const(int k) {
-    uint32_t s = 0u;
-    const uint32_t C = static_cast<uint32_t>((1 << (W - 1)) - 1) - kMagicBits;
-    for (int c = 0; c < 32; ++c)
-        if (((c * W) >> 5) == k) s += C << ((c * W) & 31);
-    return s;
-}
-
-template <int W, int C>
-__device__ __forceinline__ void run_put(uint32_t (&wd)[W], uint32_t b) {
-    constexpr int bp = C * W, k = bp >> 5, sh = bp & 31;
-    constexpr uint32_t Cn = static_cast<uint32_t>((1 << (W - 1)) - 1) - kMagicBits;
-    wd[k] += b << sh;
-    if constexpr (sh + W > 32) wd[k + 1] += (b + Cn) >> (32 - sh);
+    wd[k] += u << sh;
+    if constexpr (sh + W > 32) wd[k + 1] += u >> (32 - sh);
 }
 
 template <int W, int C>
 struct RunEncode {
-    __device__ __forceinline__ static void go(uint32_t (&wd)[W], const float2 (&xv)[16], float2 i2, float lo, float hi) {
+    __device__ __forceinline__ static void go(uint32_t (&wd)[W], const float2 (&xv)[16], float2 i2, int off, int top) {
         const float2 t = __fadd2_rn(__fmul2_rn(xv[C / 2], i2), make_float2(kMagic, kMagic));
-        run_put<W, C>(wd, __float_as_uint(fminf(fmaxf(t.x, lo), hi)));
-        run_put<W, C + 1>(wd, __float_as_uint(fminf(fmaxf(t.y, lo), hi)));
-        RunEncode<W, C + 2>::go(wd, xv, i2, lo, hi);
+        run_put<W, C>(wd, static_cast<uint32_t>(__viaddmin_s32_relu(__float_as_int(t.x), off, top)));
+        run_put<W, C + 1>(wd, static_cast<uint32_t>(__viaddmin_s32_relu(__float_as_int(t.y), off, top)));
+        RunEncode<W, C + 2>::go(wd, xv, i2, off, top);
     }
 };
 template <int W>
 struct RunEncode<W, 32> {
-    __device__ __forceinline__ static void go(uint32_t (&)[W], const float2 (&)[16], float2, float, float) {}
+    __device__ __forceinline__ static void go(uint32_t (&)[W], const float2 (&)[16], float2, int, int) {}
 };
 
 // MAXA: alignment of the row starts (16 bytes for dv = 128, 8 for dv = 64).
@@ -257,11 +194,11 @@ __device__ __forceinline__ void pack_run(const float2 (&xv)[16], float inv, uint
         }
         store_words<1, MAXA>(dst, wd);
     } else if constexpr (W >= 2) {
-        constexpr float n = static_cast<float>((1 << (W - 1)) - 1);
+        constexpr int n = (1 << (W - 1)) - 1;
         uint32_t wd[W];
 #pragma unroll
-        for (int k = 0; k < W; ++k) wd[k] = run_pack_const<W>(k);
-        RunEncode<W, 0>::go(wd, xv, make_float2(inv, inv), kMagic - n, kMagic + n);
+        for (int k = 0; k < W; ++k) wd[k] = 0u;
+        RunEncode<W, 0>::go(wd, xv, make_float2(inv, inv), n - static_cast<int>(kMagicBits), 2 * n);
         store_words<W, MAXA>(dst, wd);
     }
 }
@@ -490,8 +427,9 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
             const int w = min(static_cast<int>(S.w_in[i]), 16);
             const float D = f16_value(S.sc_in[i]);
             const float A = 8388608.0f + (w >= 2 ? sm.wc[w].x : 0.0f);
-            sm.deq[i] = make_float4(-A, (w >= 2 ? D : (w == 1 ? -2.0f * D : 0.0f)) * d,
-                                    (w == 1 ? D : 0.0f) * d, 0.0f);
+            const float Sd = (w >= 2 ? D : (w == 1 ? -2.0f * D : 0.0f)) * d, Bd = (w == 1 ? D : 0.0f) * d;
+            sm.deqAS[i] = make_float4(-A, -A, Sd, Sd);
+            sm.deqB[i] = make_float2(Bd, Bd);
             sm.a[i] = ai;
             // k . q: one partial per warp of rows
             const float kq = warp_sum(kk * S.q[i]);
@@ -547,8 +485,8 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                 const int r = r4 + rr;
                 uint32_t u[CPL];
                 extract_codes<CPL>(pay + offs[rr], lane, static_cast<int>((w4 >> (8 * rr)) & 0xFFu), u);
-                const float4 dq = sm.deq[i0 + rr];
-                const float2 A2 = make_float2(dq.x, dq.x), S2 = make_float2(dq.y, dq.y), B2 = make_float2(dq.z, dq.z);
+                const float4 as = sm.deqAS[i0 + rr];
+                const float2 A2 = make_float2(as.x, as.y), S2 = make_float2(as.z, as.w), B2 = sm.deqB[i0 + rr];
 #pragma unroll
                 for (int c = 0; c < CP2; ++c) {
                     const float2 t2 = make_float2(__uint_as_float(kTwo23Bits | u[2 * c]),
@@ -765,12 +703,13 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                 xv[2 * g2 + 1] = make_float2(v.z, v.w);
             }
             // row range R = max |x| (identical in the row's TPR lanes)
-            float lmax = 0.0f;
+            float m4[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
             for (int c = 0; c < 16; ++c) {
                 av[c] = make_float2(fabsf(xv[c].x), fabsf(xv[c].y));
-                lmax = fmaxf(lmax, fmaxf(av[c].x, av[c].y));
+                m4[c & 3] = fmaxf(m4[c & 3], fmaxf(av[c].x, av[c].y));
             }
+            const float lmax = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
             float R = lmax;
 #pragma unroll
             for (int o = 1; o < TPR; o <<= 1) R = fmaxf(R, __shfl_xor_sync(kFull, R, o));
