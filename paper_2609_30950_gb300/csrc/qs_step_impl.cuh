@@ -24,6 +24,7 @@
 #include <type_traits>
 
 #include "qs_common.cuh"
+#include "qs_head.cuh"
 
 namespace qs {
 
@@ -662,7 +663,12 @@ cudaError_t launch_step_shape(const qstate_cfg& cfg, int src_packed, int dst_pac
     QS_CASE(false, false, true)
     QS_CASE(false, true, false)
     QS_CASE(false, false, false)
-    if (DK % 32 == 0) {
+    if constexpr (HeadGeom<DK, DV>::ok) {
+        // head unit: the kernel whose lanes own whole scale groups
+        if (head && src_packed && dst_packed) return launch_head_t<DK, DV, true, true>(cfg, p, stream);
+        if (head && !src_packed && dst_packed) return launch_head_t<DK, DV, false, true>(cfg, p, stream);
+        if (head && src_packed && !dst_packed) return launch_head_t<DK, DV, true, false>(cfg, p, stream);
+    } else if (DK % 32 == 0) {
         QS_CASE(true, true, true)
         QS_CASE(true, false, true)
         QS_CASE(true, true, false)
