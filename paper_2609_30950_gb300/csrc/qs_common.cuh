@@ -99,48 +99,4 @@ __device__ __forceinline__ void extract_codes(const uint8_t* row, int lane, int 
     }
 }
 
-// Write the row's codes.  Lanes form groups of G = CPL-lane chunks whose combined width is a
-// whole number of bytes; the group's first lane writes them.  Every byte of the row is
-// written exactly once (no zero fill needed).  All 32 lanes must call this.
-template <int CPL>
-__device__ __forceinline__ void store_codes(uint8_t* row, int lane, int w, const uint32_t (&u)[CPL]) {
-    uint64_t chunk = 0;
-#pragma unroll
-    for (int c = 0; c < CPL; ++c) chunk |= static_cast<uint64_t>(u[c]) << (c * w);
-    const int cb = CPL * w;                     // bits per lane
-    // smallest G (1, 2 or 4) with G * cb a multiple of 8
-    const int G = (cb % 8 == 0) ? 1 : ((2 * cb) % 8 == 0 ? 2 : 4);
-    // gather the group's chunks into a 128-bit value (lo, hi)
-    uint64_t lo = chunk, hi = 0;
-#pragma unroll
-    for (int g = 1; g < 4; ++g) {
-        uint64_t other = __shfl_down_sync(kFull, chunk, g);
-        if (g < G) {
-            const int s = g * cb;               // 1 <= s < 128
-            if (s < 64) {
-                lo |= other << s;
-                hi |= other >> (64 - s);
-            } else {
-                hi |= other << (s - 64);
-            }
-        }
-    }
-    if ((lane % G) == 0) {
-        const int nbytes = (G * cb) >> 3;
-        uint8_t* dst = row + (lane / G) * nbytes;
-        for (int k = 0; k < nbytes; ++k) {
-            uint64_t src = (k < 8) ? lo : hi;
-            dst[k] = static_cast<uint8_t>(src >> ((k & 7) * 8));
-        }
-    }
-}
-
-// Dequantised value of code u at width w (Sec. 3 levels): w >= 2 -> (u - n) Delta,
-// w = 1 -> +-m, w = 0 -> 0.  nf2 = 2^23 + n (exact).
-__device__ __forceinline__ float dequant(uint32_t u, int w, float D, float nf2) {
-    if (w >= 2) return __fmul_rn(__fsub_rn(__uint_as_float(kTwo23Bits | u), nf2), D);
-    if (w == 1) return u ? -D : D;
-    return 0.0f;
-}
-
 }  // namespace qs

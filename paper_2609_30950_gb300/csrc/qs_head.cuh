@@ -3,7 +3,7 @@
 // Gated DeltaNet).  Also serves pack (dense -> packed), unpack (packed -> dense) and the dense
 // reference path of this unit.
 //
-// One CTA of 8 warps per (batch element, head).  Warp w owns row block w / NCS (32 key rows,
+// One CTA of NW warps per (batch element, head).  Warp w owns row block w / NCS (32 key rows,
 // exactly one scale-group row) and column slice w % NCS (CS value columns); lane l owns the CPL
 // columns cs CS + l CPL .. + CPL - 1 of those 32 rows.  So every scale group lies in one lane,
 // whole: its range, its 1-bit mean and the squared errors of its 16 candidate steps are
@@ -30,13 +30,14 @@ namespace qs {
 
 template <int DK, int DV>
 struct HeadGeom {
-    static constexpr int NW = 8;
+    static constexpr int CPL = (DK >= 128 && DV >= 128) ? 2 : 1;   // value columns per lane
     static constexpr int NB = DK / 32;     // row blocks (one scale-group row each)
-    static constexpr int NCS = NW / NB;    // column slices per row block
-    static constexpr int CS = DV / NCS;    // value columns per slice
-    static constexpr int CPL = CS / 32;    // value columns per lane
+    static constexpr int CS = 32 * CPL;    // value columns per slice (one warp)
+    static constexpr int NCS = DV / CS;    // column slices per row block
+    static constexpr int NW = NB * NCS;    // warps: 8 at 128 x 128 and 128 x 64, 4 at 64 x 64
+    static constexpr int NT = 32 * NW;
     static constexpr int NSG = NB * DV;    // scale groups per head
-    static constexpr bool ok = DK % 32 == 0 && NW % NB == 0 && CS % 32 == 0 && (CPL == 1 || CPL == 2);
+    static constexpr bool ok = DK % 32 == 0 && DV % CS == 0 && NW <= 8 && DK <= NT && DV < NT;
 };
 
 template <int DK, int DV>
@@ -73,10 +74,10 @@ __device__ __forceinline__ float2 hv_pair(float a, float b) { return make_float2
 __device__ __forceinline__ float hv_lo(float4 q) { return q.x; }
 
 template <int DK, int DV, bool SRC_PACKED, bool DST_PACKED>
-__global__ void __launch_bounds__(256, 2) head_kernel(const StepParams p) {
+__global__ void __launch_bounds__(HeadGeom<DK, DV>::NT, 2) head_kernel(const StepParams p) {
     using G = HeadGeom<DK, DV>;
     static_assert(G::ok, "head-unit layout");
-    constexpr int NB = G::NB, NCS = G::NCS, CS = G::CS, CPL = G::CPL, NSG = G::NSG;
+    constexpr int NB = G::NB, NCS = G::NCS, CS = G::CS, CPL = G::CPL, NSG = G::NSG, NT = G::NT;
     using V = typename HeadLane<CPL>::V;
     using Sm = HeadSmem<DK, DV>;
     extern __shared__ __align__(16) uint8_t smem_raw[];
@@ -115,7 +116,7 @@ __global__ void __launch_bounds__(256, 2) head_kernel(const StepParams p) {
         const Vec* src = reinterpret_cast<const Vec*>(p.in_payload + static_cast<size_t>(b) * p.region_bytes +
                                                       p.in_head_off[bh]);
         Vec* dst = reinterpret_cast<Vec*>(pay);
-        for (int i = tid; i < bytes_in / static_cast<int>(sizeof(Vec)); i += 256) dst[i] = __ldg(src + i);
+        for (int i = tid; i < bytes_in / static_cast<int>(sizeof(Vec)); i += NT) dst[i] = __ldg(src + i);
         if (tid < 4) reinterpret_cast<uint32_t*>(pay + bytes_in)[tid] = 0u;   // readable tail
     }
     if (tid < kNFit) sm.fitf[tid] = fit_factor(tid);
@@ -165,7 +166,7 @@ __global__ void __launch_bounds__(256, 2) head_kernel(const StepParams p) {
     if (SRC_PACKED) __syncthreads();   // the staging buffer is reused for the output rows
     if (DST_PACKED) {                  // zero the output rows: codes are OR-ed in
         const int nz = (bytes_out + 16) / 16;
-        for (int i = tid; i < nz; i += 256) reinterpret_cast<uint4*>(pay)[i] = make_uint4(0, 0, 0, 0);
+        for (int i = tid; i < nz; i += NT) reinterpret_cast<uint4*>(pay)[i] = make_uint4(0, 0, 0, 0);
         if (!has_tokens) __syncthreads();
     }
 
@@ -434,7 +435,7 @@ __global__ void __launch_bounds__(256, 2) head_kernel(const StepParams p) {
         __syncthreads();
         Vec* dst = reinterpret_cast<Vec*>(p.out_payload + static_cast<size_t>(b) * p.region_bytes + p.out_head_off[bh]);
         const Vec* srcv = reinterpret_cast<const Vec*>(pay);
-        for (int i = tid; i < bytes_out / static_cast<int>(sizeof(Vec)); i += 256) dst[i] = srcv[i];
+        for (int i = tid; i < bytes_out / static_cast<int>(sizeof(Vec)); i += NT) dst[i] = srcv[i];
     } else if (p.dense_out != nullptr) {
         float* dst = p.dense_out + (static_cast<size_t>(bh) * DK + r0) * DV + col0;
 #pragma unroll
@@ -459,7 +460,7 @@ cudaError_t launch_head_t(const qstate_cfg& cfg, const StepParams& p, cudaStream
     if (e != cudaSuccess) return e;
     StepParams q = p;
     q.stage_bytes = stage;
-    kern<<<cfg.B * cfg.H, 256, smem, stream>>>(q);
+    kern<<<cfg.B * cfg.H, HeadGeom<DK, DV>::NT, smem, stream>>>(q);
     return cudaGetLastError();
 }
 

@@ -1,4 +1,5 @@
-// qs_step_impl.cuh -- the fused write-back kernel of libqstate (sm_103a).
+// qs_step_impl.cuh -- general write-back kernel of libqstate for the row allocation unit (sm_103a);
+// the head unit has its own kernel (qs_head.cuh).
 //
 // One CTA per (batch element, head), 8 warps.  Warp w owns key rows [w*RPW, (w+1)*RPW); lane
 // l owns value columns [l*CPL, (l+1)*CPL) of each of them, so one row is handled by one warp
@@ -28,21 +29,19 @@
 
 namespace qs {
 
-template <int DK, int DV, bool HEAD>
+template <int DK, int DV>
 struct alignas(16) StepSmem {
     static constexpr int NW = 8;
-    static constexpr int NSG = HEAD ? (DK / 32) * DV : DK;
-    float cand[HEAD ? 1 : DK][kNFit][2];  // row unit: (Delta_k, 1/Delta_k) of the refit rows
+    static constexpr int NSG = DK;
+    float cand[DK][kNFit][2];             // (Delta_k, 1/Delta_k) of the refit rows
     float k[DK], q[DK], d[DK];
     float v[DV], u[DV];
     float ga[DK], gw[DV];                 // general erasure: this token's a and w
     float red[2][NW][DV];                 // p and r partials per warp
     float scale_in[NSG];                  // source steps / means (float)
-    float ms[DK], mr[DK];                 // EMA statistics (head unit uses [0])
+    float ms[DK], mr[DK];                 // EMA statistics per row
     float deqA[DK], deqS[DK], deqB[DK];   // row unit dequantisation constants
     float rowR[DK], rowM[DK], rowD[DK], rowInv[DK];
-    float fit_red[HEAD ? NW * 4 * DV : 1];// head unit: partial SSEs, 4 candidates per round
-    float colmax[HEAD ? NW * DV : 1];     // head unit: per-warp column maxima / sums
     float fitf[kNFit];                    // f_k = (5 + k) / 20
     float inv_n[17];                      // 1 / (2^(w-1) - 1), w = 2..16
     float wsum[4][NW];                    // per-warp partial k.q, |k|^2, a.k, |a|^2
@@ -90,10 +89,10 @@ __device__ __forceinline__ void or_codes(uint32_t* words, int lane, int w, const
     if (hi) atomicOr(words + idx + 2, hi);
 }
 
-template <int DK, int DV, bool HEAD, bool SRC_PACKED, bool DST_PACKED>
+template <int DK, int DV, bool SRC_PACKED, bool DST_PACKED>
 __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
     constexpr int NW = 8, RPW = DK / NW, CPL = DV / 32;
-    using Sm = StepSmem<DK, DV, HEAD>;
+    using Sm = StepSmem<DK, DV>;
     constexpr int NSG = Sm::NSG;
     extern __shared__ __align__(16) uint8_t smem_raw[];
     Sm& sm = *reinterpret_cast<Sm*>(smem_raw);
@@ -101,7 +100,7 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int bh = blockIdx.x, b = bh / p.H, h = bh - b * p.H;
-    const size_t ubase = HEAD ? static_cast<size_t>(bh) : static_cast<size_t>(bh) * DK;
+    const size_t ubase = static_cast<size_t>(bh) * DK;
     const size_t gbase = static_cast<size_t>(bh) * NSG;
     const bool has_tokens = p.t_end > p.t_begin;
     const bool stats = has_tokens && p.ema_s != nullptr;
@@ -114,22 +113,17 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
         sm.inv_n[w] = w >= 2 ? __frcp_rn(static_cast<float>((1 << (w - 1)) - 1)) : 0.0f;
     }
     if (SRC_PACKED) {
-        for (int i = tid; i < DK; i += 256) sm.w_in[i] = HEAD ? p.in_widths[bh] : p.in_widths[ubase + i];
+        for (int i = tid; i < DK; i += 256) sm.w_in[i] = p.in_widths[ubase + i];
         for (int g = tid; g < NSG; g += 256) sm.scale_in[g] = f16_value(p.in_scales[gbase + g]);
     }
     if (DST_PACKED) {
-        for (int i = tid; i < DK; i += 256) sm.w_out[i] = HEAD ? p.out_widths[bh] : p.out_widths[ubase + i];
+        for (int i = tid; i < DK; i += 256) sm.w_out[i] = p.out_widths[ubase + i];
         for (int g = tid; g < NSG; g += 256) sm.fidx_in[g] = p.in_fidx ? p.in_fidx[gbase + g] : 15;
     }
     if (stats) {
-        if (!HEAD) {
-            for (int i = tid; i < DK; i += 256) {
-                sm.ms[i] = p.ema_s[ubase + i];
-                sm.mr[i] = p.ema_r[ubase + i];
-            }
-        } else if (tid == 0) {
-            sm.ms[0] = p.ema_s[ubase];
-            sm.mr[0] = p.ema_r[ubase];
+        for (int i = tid; i < DK; i += 256) {
+            sm.ms[i] = p.ema_s[ubase + i];
+            sm.mr[i] = p.ema_r[ubase + i];
         }
     }
     __syncthreads();
@@ -166,7 +160,7 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
                 atomicExch(&sm.flag, 1);
         }
     }
-    if (SRC_PACKED && !HEAD && tid >= 64 && tid < 64 + DK) {
+    if (SRC_PACKED && tid >= 64 && tid < 64 + DK) {
         // per-row dequantisation x = (float(u) - A) S + Bc: w >= 2 -> (q) Delta; w = 1 -> +-m;
         // w = 0 -> 0 (float(u) is 2^23 + u built from the code bits)
         const int i = tid - 64;
@@ -204,17 +198,10 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
             const int w = sm.w_in[i];
             uint32_t u[CPL];
             extract_codes<CPL>(pay + sm.off_in[i], lane, w, u);
-            if (!HEAD) {
-                const float A = sm.deqA[i], S = sm.deqS[i], Bc = sm.deqB[i];
+            const float A = sm.deqA[i], S = sm.deqS[i], Bc = sm.deqB[i];
 #pragma unroll
-                for (int c = 0; c < CPL; ++c)
-                    x[r][c] = fmaf(__fsub_rn(__uint_as_float(kTwo23Bits | u[c]), A), S, Bc);
-            } else {
-                const float nf2 = 8388608.0f + static_cast<float>(w >= 2 ? (1 << (w - 1)) - 1 : 0);
-#pragma unroll
-                for (int c = 0; c < CPL; ++c)
-                    x[r][c] = dequant(u[c], w, sm.scale_in[(i >> 5) * DV + lane * CPL + c], nf2);
-            }
+            for (int c = 0; c < CPL; ++c)
+                x[r][c] = fmaf(__fsub_rn(__uint_as_float(kTwo23Bits | u[c]), A), S, Bc);
         } else if (p.dense_in != nullptr) {
             const float* src = p.dense_in + (static_cast<size_t>(bh) * DK + i) * DV + lane * CPL;
             if (CPL == 4) {
@@ -262,7 +249,7 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
             sm.ga[i] = ai;
             // Sec. 3 statistics per row (general erasure: after the barrier, as the erasure
             // term needs all of k)
-            if (stats && !HEAD && !p.general) {
+            if (stats && !p.general) {
                 const float xs = -expm1f(-2.0f * rate);
                 const float xr = p.erase ? __fmul_rn(__fmul_rn(beta, __fsub_rn(2.0f, beta)), __fmul_rn(kk, kk)) : 0.0f;
                 if (t == 0) {
@@ -289,7 +276,7 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
             if (p.general) sm.gw[tid] = __ldg(p.w_in + tok * DV + tid);
         }
         __syncthreads();
-        if (stats && !HEAD && p.general && tid < DK) {   // Sec. 3 statistics per row
+        if (stats && p.general && tid < DK) {   // Sec. 3 statistics per row
             const int i = tid;
             float rate = rate_h;
             if (p.decay_row)
@@ -347,31 +334,6 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
             sm.u[j] = u;
             p.o[tok * DV + j] = fmaf(u, kq, Rr);   // o = S^T q = S'^T q + u (k . q)
         }
-        if (stats && HEAD && tid == 0) {   // Sec. 3 statistics per head
-            float k2 = 0.0f;
-#pragma unroll
-            for (int w = 0; w < DK / 32; ++w) k2 += sm.wsum[1][w];
-            const float xs = -expm1f(-2.0f * rate_h);
-            float xr = p.erase ? __fmul_rn(__fmul_rn(beta, __fsub_rn(2.0f, beta)),
-                                           __fdiv_rn(k2, static_cast<float>(DK)))
-                               : 0.0f;
-            if (p.general) {   // mean over the rows of 2 a_i k_i - a_i^2 |k|^2
-                float ak = 0.0f, aa = 0.0f;
-#pragma unroll
-                for (int w = 0; w < DK / 32; ++w) {
-                    ak += sm.wsum[2][w];
-                    aa += sm.wsum[3][w];
-                }
-                xr = __fdiv_rn(__fsub_rn(__fmul_rn(2.0f, ak), __fmul_rn(aa, k2)), static_cast<float>(DK));
-            }
-            if (t == 0) {
-                sm.ms[0] = xs;
-                sm.mr[0] = xr;
-            } else {
-                sm.ms[0] = __fadd_rn(sm.ms[0], __fmul_rn(p.alpha, __fsub_rn(xs, sm.ms[0])));
-                sm.mr[0] = __fadd_rn(sm.mr[0], __fmul_rn(p.alpha, __fsub_rn(xr, sm.mr[0])));
-            }
-        }
         __syncthreads();
 #pragma unroll
         for (int r = 0; r < RPW; ++r) {
@@ -384,7 +346,7 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
     // ---- 5. write-back ------------------------------------------------------------------------
     if (DST_PACKED) {
         const bool refit = (p.fit_every <= 1) || ((p.w_index + h) % p.fit_every == 0);
-        if (!HEAD) {
+        {
             // (a) row ranges (and 1-bit means) by warp reductions
 #pragma unroll
             for (int r = 0; r < RPW; ++r) {
@@ -486,117 +448,6 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
                 }
                 or_codes<CPL>(reinterpret_cast<uint32_t*>(pay + sm.off_out[i]), lane, w, u);
             }
-        } else {
-            // head unit: one width per head; scale groups = 32 key rows x one value column.
-            // Warps 2m and 2m+1 hold the two halves of row block m.
-            const int w = sm.w_out[0];
-            const int blk = warp >> 1;
-            float* mine = sm.colmax + warp * DV;
-            const float* other = sm.colmax + (warp ^ 1) * DV;
-            float R[CPL], Dc[CPL], ic[CPL];
-            int fc[CPL];
-#pragma unroll
-            for (int c = 0; c < CPL; ++c) {
-                float m = 0.0f;
-#pragma unroll
-                for (int r = 0; r < RPW; ++r) m = (w == 1) ? m + fabsf(x[r][c]) : fmaxf(m, fabsf(x[r][c]));
-                mine[lane * CPL + c] = m;
-            }
-            __syncthreads();
-#pragma unroll
-            for (int c = 0; c < CPL; ++c) {
-                const float a = mine[lane * CPL + c], o2 = other[lane * CPL + c];
-                // same combination order in both warps of the pair: even half first
-                R[c] = (w == 1) ? ((warp & 1) ? o2 + a : a + o2) : fmaxf(a, o2);
-                fc[c] = sm.fidx_in[blk * DV + lane * CPL + c];
-            }
-            uint32_t n = 0;
-            float nf = 0.0f, inv_n = 0.0f;
-            if (w >= 2) {
-                n = (1u << (w - 1)) - 1u;
-                nf = static_cast<float>(n);
-                inv_n = sm.inv_n[w];
-            }
-            if (w >= 2 && refit) {
-                float best[CPL];
-#pragma unroll
-                for (int c = 0; c < CPL; ++c) best[c] = INFINITY;
-                float* part = sm.fit_red + warp * 4 * DV;
-                const float* opart = sm.fit_red + (warp ^ 1) * 4 * DV;
-#pragma unroll 1
-                for (int round = 0; round < 4; ++round) {
-#pragma unroll
-                    for (int kk = 0; kk < 4; ++kk) {
-                        const float f = sm.fitf[round * 4 + kk];
-#pragma unroll
-                        for (int c = 0; c < CPL; ++c) {
-                            const float D = cand_step(f, R[c], inv_n);
-                            const float inv = step_rcp(D);
-                            float acc = 0.0f;
-#pragma unroll
-                            for (int r = 0; r < RPW; ++r) {
-                                const float a = fabsf(x[r][c]);
-                                const float tq = fminf(__fadd_rn(__fmul_rn(a, inv), kMagic), kMagic + nf);
-                                const float e = fmaf(-__fsub_rn(tq, kMagic), D, a);
-                                acc = fmaf(e, e, acc);
-                            }
-                            part[kk * DV + lane * CPL + c] = acc;
-                        }
-                    }
-                    __syncthreads();
-#pragma unroll
-                    for (int kk = 0; kk < 4; ++kk) {
-#pragma unroll
-                        for (int c = 0; c < CPL; ++c) {
-                            const float a = part[kk * DV + lane * CPL + c], o2 = opart[kk * DV + lane * CPL + c];
-                            const float tot = (warp & 1) ? o2 + a : a + o2;
-                            if (R[c] == 0.0f) {
-                                fc[c] = kNFit - 1;
-                            } else if (tot <= best[c]) {
-                                best[c] = tot;
-                                fc[c] = round * 4 + kk;
-                            }
-                        }
-                    }
-                    __syncthreads();
-                }
-            }
-#pragma unroll
-            for (int c = 0; c < CPL; ++c) {
-                if (w >= 2) {
-                    Dc[c] = (R[c] == 0.0f) ? 0.0f : cand_step(sm.fitf[fc[c]], R[c], inv_n);
-                } else if (w == 1) {
-                    Dc[c] = f16_round(__fdiv_rn(R[c], 32.0f));
-                } else {
-                    Dc[c] = 0.0f;
-                }
-                ic[c] = step_rcp(Dc[c]);
-            }
-#pragma unroll
-            for (int r = 0; r < RPW; ++r) {
-                const int i = warp * RPW + r;
-                uint32_t u[CPL];
-#pragma unroll
-                for (int c = 0; c < CPL; ++c) {
-                    if (w >= 2) {
-                        const float tq = code_magic(x[r][c], ic[c], kMagic - nf, kMagic + nf);
-                        u[c] = __float_as_uint(tq) - (kMagicBits - n);
-                    } else if (w == 1) {
-                        u[c] = x[r][c] < 0.0f ? 1u : 0u;
-                    } else {
-                        u[c] = 0u;
-                    }
-                }
-                or_codes<CPL>(reinterpret_cast<uint32_t*>(pay + sm.off_out[i]), lane, w, u);
-            }
-            if ((warp & 1) == 0) {
-#pragma unroll
-                for (int c = 0; c < CPL; ++c) {
-                    const int g = blk * DV + lane * CPL + c;
-                    sm.out_scale[g] = f16_bits(Dc[c]);
-                    sm.out_fidx[g] = static_cast<uint8_t>(fc[c]);
-                }
-            }
         }
         __syncthreads();
         const int nbytes = sm.off_out[DK];
@@ -609,7 +460,7 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
             p.out_scales[gbase + g] = sm.out_scale[g];
             p.out_fidx[gbase + g] = sm.out_fidx[g];
         }
-        if (!HEAD && p.range != nullptr)
+        if (p.range != nullptr)
             for (int i = tid; i < DK; i += 256) p.range[ubase + i] = sm.rowR[i];
     } else if (p.dense_out != nullptr) {
 #pragma unroll
@@ -625,22 +476,17 @@ __global__ void __launch_bounds__(256, 2) step_kernel(const StepParams p) {
         }
     }
     if (stats) {
-        if (!HEAD) {
-            for (int i = tid; i < DK; i += 256) {
-                p.ema_s[ubase + i] = sm.ms[i];
-                p.ema_r[ubase + i] = sm.mr[i];
-            }
-        } else if (tid == 0) {
-            p.ema_s[ubase] = sm.ms[0];
-            p.ema_r[ubase] = sm.mr[0];
+        for (int i = tid; i < DK; i += 256) {
+            p.ema_s[ubase + i] = sm.ms[i];
+            p.ema_r[ubase + i] = sm.mr[i];
         }
     }
 }
 
-template <int DK, int DV, bool HEAD, bool SRC_PACKED, bool DST_PACKED>
+template <int DK, int DV, bool SRC_PACKED, bool DST_PACKED>
 cudaError_t launch_step_t(const qstate_cfg& cfg, const StepParams& p, cudaStream_t stream) {
-    auto kern = step_kernel<DK, DV, HEAD, SRC_PACKED, DST_PACKED>;
-    const size_t smem = sizeof(StepSmem<DK, DV, HEAD>) +
+    auto kern = step_kernel<DK, DV, SRC_PACKED, DST_PACKED>;
+    const size_t smem = sizeof(StepSmem<DK, DV>) +
                         ((SRC_PACKED || DST_PACKED) ? static_cast<size_t>(DK) * DV * cfg.bmax / 8 + 32 : 0);
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
@@ -656,23 +502,21 @@ cudaError_t launch_step_shape(const qstate_cfg& cfg, int src_packed, int dst_pac
                               const StepParams& p, cudaStream_t stream) {
     // the allocation unit only shapes packing: dense -> dense runs the row-unit instance
     const bool head = cfg.unit_kind == QSTATE_UNIT_HEAD && (src_packed || dst_packed);
-#define QS_CASE(HD, SP, DP)                                                            \
-    if (head == HD && (src_packed != 0) == SP && (dst_packed != 0) == DP)              \
-        return launch_step_t<DK, DV, HD, SP, DP>(cfg, p, stream);
-    QS_CASE(false, true, true)
-    QS_CASE(false, false, true)
-    QS_CASE(false, true, false)
-    QS_CASE(false, false, false)
-    if constexpr (HeadGeom<DK, DV>::ok) {
-        // head unit: the kernel whose lanes own whole scale groups
-        if (head && src_packed && dst_packed) return launch_head_t<DK, DV, true, true>(cfg, p, stream);
-        if (head && !src_packed && dst_packed) return launch_head_t<DK, DV, false, true>(cfg, p, stream);
-        if (head && src_packed && !dst_packed) return launch_head_t<DK, DV, true, false>(cfg, p, stream);
-    } else if (DK % 32 == 0) {
-        QS_CASE(true, true, true)
-        QS_CASE(true, false, true)
-        QS_CASE(true, true, false)
+    if (head) {   // head unit: the kernel whose lanes own whole scale groups
+        if constexpr (HeadGeom<DK, DV>::ok) {
+            if (src_packed && dst_packed) return launch_head_t<DK, DV, true, true>(cfg, p, stream);
+            if (!src_packed && dst_packed) return launch_head_t<DK, DV, false, true>(cfg, p, stream);
+            return launch_head_t<DK, DV, true, false>(cfg, p, stream);
+        }
+        return cudaErrorInvalidValue;
     }
+#define QS_CASE(SP, DP)                                                                \
+    if ((src_packed != 0) == SP && (dst_packed != 0) == DP)                            \
+        return launch_step_t<DK, DV, SP, DP>(cfg, p, stream);
+    QS_CASE(true, true)
+    QS_CASE(false, true)
+    QS_CASE(true, false)
+    QS_CASE(false, false)
 #undef QS_CASE
     return cudaErrorInvalidValue;
 }

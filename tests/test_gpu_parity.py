@@ -128,7 +128,20 @@ def _width_map(cfgo, rng, lo, hi):
 @pytest.mark.parametrize("name,lo,hi", [("kda_decode", 0, 16), ("tiny_kda", 0, 16),
                                         ("gdn_decode", 2, 16), ("mamba2_decode", 1, 16)])
 def test_pack_unpack_vs_oracle(qs, orc, name, lo, hi):
-    w = synth.scaled(synth.WORKLOADS[name], B=2, bmin=lo, bmax=hi)
+    _pack_unpack(qs, orc, synth.scaled(synth.WORKLOADS[name], B=2, bmin=lo, bmax=hi), lo, hi)
+
+
+# Head unit at the other supported state shapes: 128 x 64 takes the kernel whose lanes own one
+# whole scale group each (one value column per lane there), 64 x 64 the general kernel.
+HEAD_SHAPES = [(128, 64), (64, 64)]
+
+
+@pytest.mark.parametrize("dk,dv", HEAD_SHAPES)
+def test_pack_unpack_head_unit_shapes(qs, orc, dk, dv):
+    _pack_unpack(qs, orc, synth.scaled(synth.WORKLOADS["gdn_decode"], B=2, H=3, dk=dk, dv=dv), 0, 16)
+
+
+def _pack_unpack(qs, orc, w, lo, hi):
     cfgq, cfgo = qs.Config.from_workload(w), orc.Cfg.from_workload(w)
     rng = np.random.default_rng(11)
     widths, head_off = _width_map(cfgo, rng, lo, hi)
@@ -320,6 +333,15 @@ def test_quantised_lockstep(qs, orc, name):
 def test_quantised_lockstep_fit_every(qs, orc):
     w = small("kda_decode", B=2, H=4, T=10, gate_bits=0)
     _lockstep(qs, orc, w, fit_every=4)
+
+
+@pytest.mark.parametrize("dk,dv", [(128, 128)] + HEAD_SHAPES)
+@pytest.mark.parametrize("fit_every", [1, 3])
+def test_quantised_lockstep_head_unit_shapes(qs, orc, dk, dv, fit_every):
+    """Gated DeltaNet (head unit) write-backs at every state shape, refitting every write-back
+    or reusing the stored factors between refits."""
+    w = small("gdn_decode", B=2, H=4, T=8, dk=dk, dv=dv)
+    _lockstep(qs, orc, w, fit_every=fit_every)
 
 
 def test_persistent_decay_lockstep(qs, orc):
