@@ -27,10 +27,10 @@
 //       output width; and, on the last warp, the next head's metadata copies
 //   B2  -> unpack into registers (update layout),
 //       partials p = a^T S', r = q^T S'
-//   B3  -> u = beta v - p, o = r + u (k.q)
-//   B4  -> S = S' + k u^T.  Further tokens of the interval repeat from the partials, with
-//       their inputs prepared one token ahead in a second buffer (prefetched into L1 one more
-//       token ahead), so each token costs two barriers.  Then the next head's packed rows are
+//   B3  -> u = beta v - p, o = r + u (k.q); meanwhile the next token's inputs are prepared
+//       in a second buffer (from registers loaded one more token ahead)
+//   B4  -> S = S' + k u^T.  Further tokens of the interval repeat from the partials, so each
+//       token costs two barriers.  Then the next head's packed rows are
 //       copied and the state goes to the buffer
 //   B5  -> write-back (row layout), batches of rows claimed dynamically: row range R, the 16
 //       candidate steps and their squared errors (refit), codes, and each lane's packed
@@ -128,9 +128,6 @@ __device__ __forceinline__ void cp_async8(void* smem, const void* gmem) {
 __device__ __forceinline__ void cp_async4(void* smem, const void* gmem) {
     const unsigned s = static_cast<unsigned>(__cvta_generic_to_shared(smem));
     asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(s), "l"(gmem) : "memory");
-}
-__device__ __forceinline__ void prefetch_l1(const void* gmem) {
-    asm volatile("prefetch.global.L1 [%0];\n" ::"l"(gmem));
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
@@ -497,85 +494,40 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
         }
 
         // ---- tokens of the interval (Eq. 1) ----------------------------------------------------
-        // Per token: (A) the last DK threads first prepare the next token's inputs (decay, a,
-        // statistics, k.q) in the other buffer, loading them from L1 where they were prefetched
-        // one token earlier; then every warp applies the decay (tokens after the first; the
-        // first one's is folded into the dequantisation) and forms the partials p = S'^T a,
-        // r = S'^T q; B3; (B) the first DV threads take the column sums, u = w o v - p and
-        // o = r + u (k.q), while the input threads prefetch the token after next; B4;
-        // (C) S = S' + k u^T.
+        // Per token: (A) every warp applies the decay (tokens after the first; the first one's
+        // is folded into the dequantisation) and forms the partials p = S'^T a, r = S'^T q; B3;
+        // (B) the first DV threads take the column sums, u = w o v - p and o = r + u (k.q),
+        // while the last DK threads prepare the next token's inputs (decay, a, statistics, k.q)
+        // in the other buffer from raw values loaded into registers one token earlier, and load
+        // the raw values of the token after next; B4; (C) S = S' + k u^T (and, under general
+        // erasure, the next token's erasure statistic, which needs all of its k).
         constexpr int P0 = NW * 32 - DK;   // first thread of the input-preparing role
         static_assert(P0 >= DV, "the two roles of the middle phase overlap");
         const int pi = tid - P0;
         const bool prep_k = pi >= 0, prep_v = pi >= 0 && pi < DV;
-        // Token inputs are pulled into L1 one token ahead of their loads (prefetches hold no
-        // registers; the loads then hit L1).  The per-token stride of every input is H rows.
-        auto prefetch = [&](const float* kp, const float* qp, const void* sp, const float* bp,
-                            const float* vp) {
-            prefetch_l1(kp);
-            prefetch_l1(qp);
-            if (p.decay_row || pi == 0) prefetch_l1(sp);
-            if (p.erase && pi == 0) prefetch_l1(bp);
-            if (prep_v) prefetch_l1(vp);
-        };
-        if (prep_k && p.t_begin + 1 < p.t_end) {
-            const size_t tn = tok0 + p.H;
+        // A preparing thread holds the raw inputs of one token in registers (its row's k, q,
+        // rate or rate code, a; beta; its column's v, w): right after preparing token t + 1 it
+        // loads token t + 2's, so the loads have a whole token to arrive.  The per-token stride
+        // of every input is H rows.
+        float rk = 0.0f, rq = 0.0f, rs = 0.0f, rbeta = 1.0f, rv = 0.0f, ra = 0.0f, rw = 0.0f;
+        int rc = 0;
+        auto load_raw = [&](size_t tn) {
+            rk = __ldg(p.k + tn * DK + pi);
+            rq = __ldg(p.q + tn * DK + pi);
             const size_t si = p.decay_row ? tn * DK + pi : tn;
-            prefetch(p.k + tn * DK + pi, p.q + tn * DK + pi,
-                     p.s_code ? static_cast<const void*>(p.s_code + si) : static_cast<const void*>(p.s + si),
-                     p.beta + tn, p.v + tn * DV + pi);
-        }
+            if (p.s_code) rc = p.s_code[si];
+            else rs = __ldg(p.s + si);
+            if (p.erase) rbeta = __ldg(p.beta + tn);
+            if (p.general) ra = __ldg(p.a_in + tn * DK + pi);
+            if (prep_v) {
+                rv = __ldg(p.v + tn * DV + pi);
+                if (p.general) rw = __ldg(p.w_in + tn * DV + pi);
+            }
+        };
+        if (prep_k && p.t_begin + 1 < p.t_end) load_raw(tok0 + p.H);
         for (int t = p.t_begin, j = 0; t < p.t_end; ++t, ++j) {
             const size_t tok = (static_cast<size_t>(b) * T + t) * p.H + h;
             const int cb = j & 1, k3 = j % 3;
-            if (prep_k && t + 1 < p.t_end) {
-                // the next token's inputs into buffer cb ^ 1, whose contents (the previous
-                // token's) were last read before the previous B4.  k goes to the third k
-                // buffer: the previous token's k is read after that B4, the one before it was
-                // last read before the previous B3.
-                const int i = pi, nb = cb ^ 1, nk3 = k3 == 2 ? 0 : k3 + 1;
-                const size_t tn = tok + p.H;   // token t + 1 of this head
-                const float* kp = p.k + tn * DK + i;
-                const float* qp = p.q + tn * DK + i;
-                const float* vp = p.v + tn * DV + i;
-                const float* bp = p.beta + tn;
-                const size_t si = p.decay_row ? tn * DK + i : tn;
-                const float nbeta = p.erase ? __ldg(bp) : 1.0f;
-                const float nk = __ldg(kp), nq = __ldg(qp);
-                float rate;
-                if (p.s_code) {
-                    const int code = min(static_cast<int>(p.s_code[si]), p.L - 1);
-                    if (p.decay_row)
-                        rate = p.L <= 4 ? S.lut[i * p.L + code]
-                                        : __ldg(p.s_lut + (static_cast<size_t>(h) * DK + i) * p.L + code);
-                    else
-                        rate = __ldg(p.s_lut + static_cast<size_t>(h) * p.L + code);
-                } else {
-                    rate = __ldg(p.s + si);
-                }
-                if (!(rate > 0.0f) || !(rate < INFINITY)) raise_status(p.status, QS_DEV_RATE);
-                (nk3 == 0 ? S.k : nk3 == 1 ? sm.tk : sm.tk2)[i] = nk;
-                (nb ? sm.tq : S.q)[i] = nq;
-                (nb ? sm.d1 : sm.d)[i] = expf(-rate);
-                (nb ? sm.a1 : sm.a)[i] = p.general ? __ldg(p.a_in + tn * DK + i) : __fmul_rn(nbeta, nk);
-                if (prep_v) {
-                    (nb ? sm.tv : S.v)[i] = __ldg(vp);
-                    if (p.general) (nb ? sm.tw : S.gw)[i] = __ldg(p.w_in + tn * DV + i);
-                }
-                if (i == 0) sm.tbeta[nb] = nbeta;
-                if (stats) {
-                    const float xs = -expm1f(-2.0f * rate);
-                    if (p.general) {
-                        sm.rowR[i] = xs;   // the erasure term needs all of the next k: after B3
-                    } else {
-                        const float xr = p.erase ? __fmul_rn(__fmul_rn(nbeta, __fsub_rn(2.0f, nbeta)), __fmul_rn(nk, nk)) : 0.0f;
-                        S.ms[i] = __fadd_rn(S.ms[i], __fmul_rn(p.alpha, __fsub_rn(xs, S.ms[i])));
-                        S.mr[i] = __fadd_rn(S.mr[i], __fmul_rn(p.alpha, __fsub_rn(xr, S.mr[i])));
-                    }
-                }
-                const float s2 = warp_sum(nk * nq);
-                if (lane == 0) sm.wsum[nb][i >> 5] = s2;
-            }
             const float* kv = k3 == 0 ? S.k : k3 == 1 ? sm.tk : sm.tk2;
             const float* qv = cb ? sm.tq : S.q;
             const float* av = cb ? sm.a1 : sm.a;
@@ -636,23 +588,56 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                 sm.u[jv] = uu;
                 p.o[tok * DV + jv] = fmaf(uu, kq, Rr);
             } else if (prep_k && t + 1 < p.t_end) {
-                if (t + 2 < p.t_end) {   // the token after next, into L1
-                    const size_t tn = tok + 2 * static_cast<size_t>(p.H);
-                    const size_t si = p.decay_row ? tn * DK + pi : tn;
-                    prefetch(p.k + tn * DK + pi, p.q + tn * DK + pi,
-                             p.s_code ? static_cast<const void*>(p.s_code + si) : static_cast<const void*>(p.s + si),
-                             p.beta + tn, p.v + tn * DV + pi);
+                // the next token's inputs into buffer cb ^ 1, whose contents (the previous
+                // token's) were last read before the previous B4.  k goes to the third k
+                // buffer: this token's k is read after the coming B4, the previous token's was
+                // last read before this token's B3.
+                const int i = pi, nb = cb ^ 1, nk3 = k3 == 2 ? 0 : k3 + 1;
+                const float nbeta = rbeta, nk = rk, nq = rq;
+                float rate;
+                if (p.s_code) {
+                    const int code = min(rc, p.L - 1);
+                    if (p.decay_row)
+                        rate = p.L <= 4 ? S.lut[i * p.L + code]
+                                        : __ldg(p.s_lut + (static_cast<size_t>(h) * DK + i) * p.L + code);
+                    else
+                        rate = __ldg(p.s_lut + static_cast<size_t>(h) * p.L + code);
+                } else {
+                    rate = rs;
                 }
-                if (p.general && stats) {
-                    // the general erasure statistic of the next token (needs all of its k)
-                    const int nk3 = k3 == 2 ? 0 : k3 + 1;
-                    const float* kb = nk3 == 0 ? S.k : nk3 == 1 ? sm.tk : sm.tk2;
-                    const float xr = general_erasure<DK>((cb ? sm.a : sm.a1)[pi], kb[pi], kb);
-                    S.ms[pi] = __fadd_rn(S.ms[pi], __fmul_rn(p.alpha, __fsub_rn(sm.rowR[pi], S.ms[pi])));
-                    S.mr[pi] = __fadd_rn(S.mr[pi], __fmul_rn(p.alpha, __fsub_rn(xr, S.mr[pi])));
+                if (!(rate > 0.0f) || !(rate < INFINITY)) raise_status(p.status, QS_DEV_RATE);
+                (nk3 == 0 ? S.k : nk3 == 1 ? sm.tk : sm.tk2)[i] = nk;
+                (nb ? sm.tq : S.q)[i] = nq;
+                (nb ? sm.d1 : sm.d)[i] = expf(-rate);
+                (nb ? sm.a1 : sm.a)[i] = p.general ? ra : __fmul_rn(nbeta, nk);
+                if (prep_v) {
+                    (nb ? sm.tv : S.v)[i] = rv;
+                    if (p.general) (nb ? sm.tw : S.gw)[i] = rw;
                 }
+                if (i == 0) sm.tbeta[nb] = nbeta;
+                if (stats) {
+                    const float xs = -expm1f(-2.0f * rate);
+                    if (p.general) {
+                        sm.rowR[i] = xs;   // the erasure term needs all of the next k: after B4
+                    } else {
+                        const float xr = p.erase ? __fmul_rn(__fmul_rn(nbeta, __fsub_rn(2.0f, nbeta)), __fmul_rn(nk, nk)) : 0.0f;
+                        S.ms[i] = __fadd_rn(S.ms[i], __fmul_rn(p.alpha, __fsub_rn(xs, S.ms[i])));
+                        S.mr[i] = __fadd_rn(S.mr[i], __fmul_rn(p.alpha, __fsub_rn(xr, S.mr[i])));
+                    }
+                }
+                const float s2 = warp_sum(nk * nq);
+                if (lane == 0) sm.wsum[nb][i >> 5] = s2;
+                if (t + 2 < p.t_end) load_raw(tok + 2 * static_cast<size_t>(p.H));
             }
             __syncthreads();                                                           // B4
+            if (prep_k && t + 1 < p.t_end && p.general && stats) {
+                // the general erasure statistic of the next token (needs all of its k)
+                const int nk3 = k3 == 2 ? 0 : k3 + 1;
+                const float* kb = nk3 == 0 ? S.k : nk3 == 1 ? sm.tk : sm.tk2;
+                const float xr = general_erasure<DK>((cb ? sm.a : sm.a1)[pi], kb[pi], kb);
+                S.ms[pi] = __fadd_rn(S.ms[pi], __fmul_rn(p.alpha, __fsub_rn(sm.rowR[pi], S.ms[pi])));
+                S.mr[pi] = __fadd_rn(S.mr[pi], __fmul_rn(p.alpha, __fsub_rn(xr, S.mr[pi])));
+            }
             float2 u2[CP2];
 #pragma unroll
             for (int c = 0; c < CP2; ++c) u2[c] = reinterpret_cast<const float2*>(&sm.u[lane * CPL])[c];
