@@ -69,12 +69,14 @@ __device__ int block_exclusive_scan(int v, int* red, int* total) {
 }  // namespace
 
 // Allocation weight c_u (Eq. 3 and the alternatives of Table 1), one IEEE rounding per
-// operation.  Rs / gmean: the batch element's ranges and group means of R^2 (row unit).
-__device__ float weight(const AllocParams& p, int u, size_t base, const float* Rs, const float* gmean, int gsz) {
+// operation.  ms_s / mr_s: the batch element's EMA statistics; Rs / gmean: its ranges, stored
+// with one padding word after every group of gsz units, and the group means of R^2 (row unit).
+__device__ float weight(const AllocParams& p, int u, const float* ms_s, const float* mr_s, const float* Rs,
+                        const float* gmean, int gsz) {
     const int kind = p.weight_kind;
     float R2 = 1.0f, rt2 = 1.0f;   // R^2 and Rtilde^2 (1 for the head unit)
     if (p.unit_row) {
-        const float R = Rs[u];
+        const float R = Rs[u + u / gsz];
         R2 = __fmul_rn(R, R);
         const float m = gmean[u / gsz];
         if (m > 0.0f) rt2 = __fdiv_rn(R2, m);
@@ -85,7 +87,7 @@ __device__ float weight(const AllocParams& p, int u, size_t base, const float* R
     const int us = kind == QSTATE_WEIGHT_SHUFFLE
                        ? static_cast<int>((static_cast<long long>(p.shuf_a) * u + p.shuf_b) % p.units)
                        : u;
-    const float ms = p.ema_s[base + us];
+    const float ms = ms_s[us];
     if (kind == QSTATE_WEIGHT_PERSIST) return __fmul_rn(__fdiv_rn(1.0f, ms), rt2);
     if (kind == QSTATE_WEIGHT_WBFACTOR) {
         float pw = 1.0f, bb = __fsub_rn(1.0f, ms);   // (1 - m_s)^C, low bit first
@@ -95,7 +97,7 @@ __device__ float weight(const AllocParams& p, int u, size_t base, const float* R
         }
         return __fmul_rn(__fdiv_rn(1.0f, __fsub_rn(1.0f, pw)), rt2);
     }
-    float mr = kind == QSTATE_WEIGHT_NOERASE ? 0.0f : p.ema_r[base + us];
+    float mr = kind == QSTATE_WEIGHT_NOERASE ? 0.0f : mr_s[us];
     if (mr < 0.0f) mr = 0.0f;
     const float G = __fdiv_rn(__fsub_rn(1.0f, ms), __fadd_rn(expm1_series(mr, p.e1), ms));
     if (kind == QSTATE_WEIGHT_GAMMA_RAW) return __fmul_rn(G, R2);
@@ -147,8 +149,11 @@ __global__ void __launch_bounds__(kThreads, 2) alloc_kernel(const AllocParams p)
     int* key = reinterpret_cast<int*>(smem);
     const int gsz = p.group_heads * p.dk;
     const int ngroups = p.unit_row ? N / gsz : 0;
-    float* Rs = reinterpret_cast<float*>(key + N);                   // row unit: ranges
-    float* gmean = Rs + (p.unit_row ? N : 0);
+    float* ms_s = reinterpret_cast<float*>(key + N);                 // EMA statistics
+    float* mr_s = ms_s + N;
+    float* Rs = mr_s + N;                                              // row unit: ranges, a padding
+                                                                       // word after each group
+    float* gmean = Rs + (p.unit_row ? N + ngroups : 0);
     int* hist = reinterpret_cast<int*>(gmean + ((ngroups + 3) & ~3));
     int* redi = hist + 1024;                                           // hist: 256 bins, then H head sizes
     int* sel = redi + 72;                                              // H*, rank, low prefix
@@ -156,16 +161,25 @@ __global__ void __launch_bounds__(kThreads, 2) alloc_kernel(const AllocParams p)
     const int tid = threadIdx.x;
     const size_t base = static_cast<size_t>(blockIdx.x) * N;
 
-    // 1. mean R^2 of each output-normalisation group, summed in row order (row unit); the
-    //    ranges are staged in shared memory first so the sequential sums read on-chip data
-    if (!p.uniform && p.unit_row) {
-        for (int u = tid; u < N; u += kThreads) Rs[u] = p.range[base + u];
+    // 1. statistics and ranges staged in shared memory (independent coalesced loads); mean R^2
+    //    of each output-normalisation group, summed in row order (row unit).  Group g's ranges
+    //    sit at stride gsz + 1, so the threads summing different groups in lockstep hit
+    //    different banks.
+    if (!p.uniform) {
+        for (int u = tid; u < N; u += kThreads) {
+            ms_s[u] = p.ema_s[base + u];
+            mr_s[u] = p.ema_r[base + u];
+            if (p.unit_row) Rs[u + u / gsz] = p.range[base + u];
+        }
         __syncthreads();
-        for (int g = tid; g < ngroups; g += kThreads) {
-            float acc = 0.0f;
+        if (p.unit_row) {
+            for (int g = tid; g < ngroups; g += kThreads) {
+                const float* rg = Rs + g * (gsz + 1);
+                float acc = 0.0f;
 #pragma unroll 8
-            for (int r = g * gsz; r < (g + 1) * gsz; ++r) acc = __fadd_rn(acc, __fmul_rn(Rs[r], Rs[r]));
-            gmean[g] = __fdiv_rn(acc, static_cast<float>(gsz));
+                for (int r = 0; r < gsz; ++r) acc = __fadd_rn(acc, __fmul_rn(rg[r], rg[r]));
+                gmean[g] = __fdiv_rn(acc, static_cast<float>(gsz));
+            }
         }
     }
     for (int k = tid; k < 256; k += kThreads) hist[k] = 0;
@@ -178,7 +192,7 @@ __global__ void __launch_bounds__(kThreads, 2) alloc_kernel(const AllocParams p)
     const long long M = p.total - static_cast<long long>(N) * p.bmin;
     for (int u = tid; u < N; u += kThreads) {
         float c = 1.0f;
-        if (!p.uniform) c = weight(p, u, base, Rs, gmean, gsz);
+        if (!p.uniform) c = weight(p, u, ms_s, mr_s, Rs, gmean, gsz);
         if (c > 0x1p60f) c = 0x1p60f;
         const int k = (c >= 0x1p-60f) ? __float_as_int(c) : kNullKey;
         key[u] = k;
@@ -317,7 +331,7 @@ __global__ void __launch_bounds__(kThreads, 2) alloc_kernel(const AllocParams p)
 
 cudaError_t launch_alloc(const AllocParams& p, cudaStream_t stream) {
     const int ngroups = p.unit_row ? p.units / (p.group_heads * p.dk) : 0;
-    const size_t smem = static_cast<size_t>(p.units) * 4 + (p.unit_row ? p.units * 4 : 0) +
+    const size_t smem = static_cast<size_t>(p.units) * 4 * 3 + (p.unit_row ? (p.units + ngroups) * 4 : 0) +
                         ((ngroups + 3) & ~3) * 4 + 1024 * 4 + 72 * 4 + 4 * 4 + p.units + 16;
     cudaError_t e = cudaFuncSetAttribute(alloc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
