@@ -528,14 +528,20 @@ int qstate_scan_host(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong,
     int in_pong = 0, w = w_index0;
     cudaError_t e = cudaSuccess;
     cudaEvent_t ev_in = nullptr, ev_out = nullptr;
-    for (int c0 = t_begin; c0 < t_end && e == cudaSuccess && rc == QSTATE_OK; c0 += chunk) {
-        const int c1 = c0 + chunk < t_end ? c0 + chunk : t_end;
+    // Inputs of chunk c + 1 are queued on the copy stream before the readouts of chunk c, so
+    // they move while chunk c computes (they fill other tokens of the device buffers); the
+    // readouts of chunk c follow once it is done.
+    auto stage_inputs = [&](int c0, int c1) {
         for (const Item& it : in)
             if (it.h && e == cudaSuccess) e = copy_tokens(it.d, it.h, it.per, c0, c1, cudaMemcpyHostToDevice);
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev_in, cudaEventDisableTiming);
         if (e == cudaSuccess) e = cudaEventRecord(ev_in, ts);
-        if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, ev_in, 0);
-        if (ev_in) cudaEventDestroy(ev_in);
+    };
+    if (t_begin < t_end) stage_inputs(t_begin, t_begin + chunk < t_end ? t_begin + chunk : t_end);
+    for (int c0 = t_begin; c0 < t_end && e == cudaSuccess && rc == QSTATE_OK; c0 += chunk) {
+        const int c1 = c0 + chunk < t_end ? c0 + chunk : t_end;
+        e = cudaStreamWaitEvent(cs, ev_in, 0);
+        cudaEventDestroy(ev_in);
         ev_in = nullptr;
         if (e != cudaSuccess) break;
         int flip = 0;
@@ -548,13 +554,15 @@ int qstate_scan_host(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong,
             dst = tmp;
             in_pong ^= 1;
         }
-        e = cudaEventCreateWithFlags(&ev_out, cudaEventDisableTiming);
+        if (c1 < t_end) stage_inputs(c1, c1 + chunk < t_end ? c1 + chunk : t_end);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev_out, cudaEventDisableTiming);
         if (e == cudaSuccess) e = cudaEventRecord(ev_out, cs);
         if (e == cudaSuccess) e = cudaStreamWaitEvent(ts, ev_out, 0);
         if (ev_out) cudaEventDestroy(ev_out);
         ev_out = nullptr;
         if (e == cudaSuccess) e = copy_tokens(o_host, o_dev, H * cfg->dv * f4, c0, c1, cudaMemcpyDeviceToHost);
     }
+    if (ev_in) cudaEventDestroy(ev_in);
     // the compute stream completes only after the last readout copy
     if (e == cudaSuccess && rc == QSTATE_OK) {
         e = cudaEventCreateWithFlags(&ev_out, cudaEventDisableTiming);
