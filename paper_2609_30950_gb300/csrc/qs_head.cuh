@@ -1,7 +1,7 @@
 // qs_head.cuh -- write-back kernel for the head allocation unit (sm_103a): one width per head and
 // one FP16 step per scale group of 32 key rows x 1 value column (Sec. 3, "Allocation units";
-// Gated DeltaNet).  Also serves pack (dense -> packed), unpack (packed -> dense) and the dense
-// reference path of this unit.
+// Gated DeltaNet).  Also serves pack (dense -> packed) and unpack (packed -> dense) for this unit;
+// the dense reference path runs the general kernel.
 //
 // One CTA of NW warps per (batch element, head).  Warp w owns row block w / NCS (32 key rows,
 // exactly one scale-group row) and column slice w % NCS (CS value columns); lane l owns the CPL
@@ -70,8 +70,6 @@ __device__ __forceinline__ float hv_get(float2 v, int c) { return c == 0 ? v.x :
 __device__ __forceinline__ float hv_get(float v, int) { return v; }
 __device__ __forceinline__ void hv_set(float2& v, int c, float s) { if (c == 0) v.x = s; else v.y = s; }
 __device__ __forceinline__ void hv_set(float& v, int, float s) { v = s; }
-__device__ __forceinline__ float2 hv_pair(float a, float b) { return make_float2(a, b); }
-__device__ __forceinline__ float hv_lo(float4 q) { return q.x; }
 
 template <int DK, int DV, bool SRC_PACKED, bool DST_PACKED>
 __global__ void __launch_bounds__(HeadGeom<DK, DV>::NT, 2) head_kernel(const StepParams p) {

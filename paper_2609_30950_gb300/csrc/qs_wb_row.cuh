@@ -6,9 +6,10 @@
 // Each CTA (NW = 8 warps, two CTAs per SM so that one's barriers and latencies overlap the
 // other's work) walks a contiguous block of heads.  While it works on head g, cp.async copies
 // head g + 1's metadata into the other half of a double buffer (widths in/out, FP16 scales,
-// fitted-factor indices, EMA statistics, the first token's k, q, v, rates and their level table)
-// and, once head g's tokens are done, head g + 1's packed rows into the single payload buffer
-// (their byte window comes from offsets fetched one head earlier).
+// fitted-factor indices, EMA statistics, the first token's k, q, v, rates and their level
+// table; issued by the one warp without a prep role) and, once head g's tokens are done, head
+// g + 1's packed rows into the single payload buffer (their byte window comes from offsets
+// fetched one head earlier).
 //
 // Two thread layouts share the head's FP32 state:
 //  * update layout: warp w owns key rows [w RPW, (w+1) RPW), lane l the value columns
@@ -30,8 +31,8 @@
 //   B3  -> u = beta v - p, o = r + u (k.q); meanwhile the next token's inputs are prepared
 //       in a second buffer (from registers loaded one more token ahead)
 //   B4  -> S = S' + k u^T.  Further tokens of the interval repeat from the partials, so each
-//       token costs two barriers.  Then the next head's packed rows are
-//       copied and the state goes to the buffer
+//       token costs two barriers.  Then the next head's packed rows are copied in and the
+//       state goes to the shared buffer
 //   B5  -> write-back (row layout), batches of rows claimed dynamically: row range R, the 16
 //       candidate steps and their squared errors (refit), codes, and each lane's packed
 //       words stored to the output region
