@@ -77,3 +77,74 @@ def test_allocation_lowers_readout_error(qs, orc, C, bbar, bmin, bmax, T, ratio)
     e_orc = float(np.sum((o_orc.astype(np.float64) - o_ref) ** 2) / np.sum(o_ref ** 2))
     print(f"oracle, Eq. 3 widths: {e_orc:.4e}")
     assert abs(errs["ours"] - e_orc) <= 0.05 * e_orc, (errs["ours"], e_orc)
+
+
+def _fp32_readouts_with_rates(qs, w, inp, s_code=None, s_lut=None, g=0):
+    """The library's unquantised recurrence, with exact rates or with coded rates + levels."""
+    cfg = qs.Config.from_workload(w, gate_bits=g)
+    d = {k: torch.from_numpy(v).cuda() for k, v in inp.items()}
+    if s_code is None:
+        X = qs.Inputs(d["q"], d["k"], d["v"], d["s"], None, None, d["beta"], w.T)
+    else:
+        X = qs.Inputs(d["q"], d["k"], d["v"], None, s_code, s_lut, d["beta"], w.T)
+    S = torch.zeros((w.B, w.H, w.dk, w.dv), dtype=torch.float32, device="cuda")
+    o = torch.zeros((w.B, w.T, w.H, w.dv), dtype=torch.float32, device="cuda")
+    qs.qstate_scan_fp32(cfg, S, X, 0, w.T, o)
+    qs.qstate_check()
+    return o.cpu().numpy().astype(np.float64)
+
+
+def test_log_uniform_gates_keep_readouts(qs, orc):
+    """Sec. 3, "Decay-gate quantization": with rates spanning decades (KDA inputs, s =
+    softplus(N(-2, 1)) drawn every token), levels uniform in log s keep the readouts of the
+    unquantised state far closer to the exact-rate recurrence than levels uniform in s
+    between the same per-channel extremes.  The library's log-uniform quantiser feeds the
+    recurrence; the linear levels, a comparison point only, are built here."""
+    w = synth.scaled(synth.WORKLOADS["kda_decode"], B=2, H=2, T=256, gate_bits=0)
+    inp = synth.host_inputs(w)
+    nchan = w.H * w.dk
+    ref = _fp32_readouts_with_rates(qs, w, inp)
+    den = np.sum(ref ** 2)
+    s_dev = torch.from_numpy(inp["s"]).cuda()
+    errs = {}
+    for g in (2, 4):
+        cfg = qs.Config.from_workload(w, gate_bits=g)
+        L = 1 << g
+        codes = torch.zeros(s_dev.shape, dtype=torch.uint8, device="cuda")
+        lut = torch.zeros(nchan * L, dtype=torch.float32, device="cuda")
+        thr = torch.zeros(nchan * (L - 1), dtype=torch.float32, device="cuda")
+        qs.qstate_quant_decay(cfg, s_dev, codes, lut, thr)
+        o = _fp32_readouts_with_rates(qs, w, inp, codes, lut, g)
+        errs[f"log g={g}"] = float(np.sum((o - ref) ** 2) / den)
+        # linear levels between the same per-channel extremes, thresholds at the midpoints
+        ss = inp["s"].reshape(-1, nchan).astype(np.float64)
+        lo, hi = ss.min(0), ss.max(0)
+        lev = lo[None, :] + (hi - lo)[None, :] * (np.arange(L)[:, None] / (L - 1))
+        th = 0.5 * (lev[1:] + lev[:-1])
+        c = (ss[:, None, :] >= th[None]).sum(1).astype(np.uint8).reshape(inp["s"].shape)
+        lin_lut = np.ascontiguousarray(lev.T.astype(np.float32)).reshape(-1)
+        o = _fp32_readouts_with_rates(qs, w, inp, torch.from_numpy(c).cuda(),
+                                      torch.from_numpy(lin_lut).cuda(), g)
+        errs[f"linear g={g}"] = float(np.sum((o - ref) ** 2) / den)
+    print("relative readout MSE:", ", ".join(f"{k} {v:.4e}" for k, v in errs.items()))
+    # the oracle's FP64 recurrence gives 2.6e-2 / 0.197 (g = 2) and 9.9e-4 / 2.0e-3 (g = 4)
+    assert errs["log g=2"] < 0.25 * errs["linear g=2"], errs
+    assert errs["log g=4"] < errs["linear g=4"], errs
+    assert errs["log g=4"] < 0.1 * errs["log g=2"], errs
+    # the same error from the oracle's quantiser and FP64 recurrence
+    c_ref, l_ref, _ = orc.quant_decay(inp["s"], nchan, 2)
+    cfgo = orc.Cfg.from_workload(w)
+    sq = l_ref[np.arange(nchan)[None, None, :], c_ref.reshape(w.B, w.T, nchan)].reshape(inp["s"].shape)
+    x = dict(inp)
+    x["s"] = sq.astype(np.float32)
+    e = 0.0
+    ref64 = np.zeros_like(ref)
+    for b in range(w.B):
+        for h in range(w.H):
+            o64, _ = orc.recur(np.zeros((w.dk, w.dv)), *orc.expand_inputs(cfgo, x, b, h), dtype=np.float64)
+            r64, _ = orc.recur(np.zeros((w.dk, w.dv)), *orc.expand_inputs(cfgo, inp, b, h), dtype=np.float64)
+            e += np.sum((o64 - r64) ** 2)
+            ref64[b, :, h] = r64
+    e_orc = e / np.sum(ref64 ** 2)
+    print(f"oracle, log g=2: {e_orc:.4e}")
+    assert abs(errs["log g=2"] - e_orc) <= 0.01 * e_orc, (errs["log g=2"], e_orc)
