@@ -471,7 +471,29 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
         }
 
         // ---- unpack + dequantise into the update layout (first token's decay folded in) -------
-        float2 x[RPW][CP2];
+        // At dv = 128 lane l holds columns 4l..4l+3 of the warp's RPW rows.  At dv = 64 the two
+        // half-warps take alternate rows (RS = 2) and lane l columns 4 (l % 16)..+3, so a lane
+        // still decodes four codes per row it visits; the partials are combined across the
+        // halves with one shuffle per value.
+        constexpr int RS = DV == 128 ? 1 : 2, NSL = RPW / RS;
+        const int half = lane / (32 / RS), cl = lane % (32 / RS);
+        float2 x[NSL][2];
+        if constexpr (RS == 2) {
+#pragma unroll
+            for (int jr = 0; jr < NSL; ++jr) {
+                const int i = warp * RPW + jr * RS + half;
+                uint32_t u[4];
+                extract_codes<4>(pay + sm.off_in[i], cl, static_cast<int>(S.w_in[i]), u);
+                const float4 as = sm.deqAS[i];
+                const float2 A2 = make_float2(as.x, as.y), S2 = make_float2(as.z, as.w), B2 = sm.deqB[i];
+#pragma unroll
+                for (int c = 0; c < 2; ++c) {
+                    const float2 t2 = make_float2(__uint_as_float(kTwo23Bits | u[2 * c]),
+                                                  __uint_as_float(kTwo23Bits | u[2 * c + 1]));
+                    x[jr][c] = __ffma2_rn(__fadd2_rn(t2, A2), S2, B2);
+                }
+            }
+        } else {
 #pragma unroll
         for (int r4 = 0; r4 < RPW; r4 += 4) {
             const int i0 = warp * RPW + r4;
@@ -492,6 +514,7 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                     x[r][c] = __ffma2_rn(__fadd2_rn(t2, A2), S2, B2);
                 }
             }
+        }
         }
 
         // ---- tokens of the interval (Eq. 1) ----------------------------------------------------
@@ -532,7 +555,15 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
             const float* kv = k3 == 0 ? S.k : k3 == 1 ? sm.tk : sm.tk2;
             const float* qv = cb ? sm.tq : S.q;
             const float* av = cb ? sm.a1 : sm.a;
-            if (j > 0) {
+            if (j > 0 && RS == 2) {
+                const float* dd = cb ? sm.d1 : sm.d;
+#pragma unroll
+                for (int jr = 0; jr < NSL; ++jr) {
+                    const float d = dd[warp * RPW + jr * RS + half];
+                    x[jr][0] = __fmul2_rn(x[jr][0], make_float2(d, d));
+                    x[jr][1] = __fmul2_rn(x[jr][1], make_float2(d, d));
+                }
+            } else if (j > 0) {
                 const float* dd = cb ? sm.d1 : sm.d;
 #pragma unroll
                 for (int r4 = 0; r4 < RPW; r4 += 4) {
@@ -546,9 +577,35 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                     }
                 }
             }
-            float2 pp[CP2], rr[CP2];
+            float2 pp[2], rr[2];
 #pragma unroll
-            for (int c = 0; c < CP2; ++c) pp[c] = rr[c] = make_float2(0.0f, 0.0f);
+            for (int c = 0; c < 2; ++c) pp[c] = rr[c] = make_float2(0.0f, 0.0f);
+            if constexpr (RS == 2) {
+#pragma unroll
+                for (int jr = 0; jr < NSL; ++jr) {
+                    const int i = warp * RPW + jr * RS + half;
+                    const float a = av[i], qq = qv[i];
+#pragma unroll
+                    for (int c = 0; c < 2; ++c) {
+                        pp[c] = __ffma2_rn(x[jr][c], make_float2(a, a), pp[c]);
+                        rr[c] = __ffma2_rn(x[jr][c], make_float2(qq, qq), rr[c]);
+                    }
+                }
+#pragma unroll
+                for (int c = 0; c < 2; ++c) {   // the other half-warp's rows
+                    pp[c].x += __shfl_xor_sync(kFull, pp[c].x, 16);
+                    pp[c].y += __shfl_xor_sync(kFull, pp[c].y, 16);
+                    rr[c].x += __shfl_xor_sync(kFull, rr[c].x, 16);
+                    rr[c].y += __shfl_xor_sync(kFull, rr[c].y, 16);
+                }
+                if (half == 0) {
+#pragma unroll
+                    for (int c = 0; c < 2; ++c) {
+                        reinterpret_cast<float2*>(&sm.rc.red[0][warp][cl * 4])[c] = pp[c];
+                        reinterpret_cast<float2*>(&sm.rc.red[1][warp][cl * 4])[c] = rr[c];
+                    }
+                }
+            } else {
 #pragma unroll
             for (int r4 = 0; r4 < RPW; r4 += 4) {
                 const float4 a4 = *reinterpret_cast<const float4*>(&av[warp * RPW + r4]);
@@ -568,6 +625,7 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
             for (int c = 0; c < CP2; ++c) {
                 reinterpret_cast<float2*>(&sm.rc.red[0][warp][lane * CPL])[c] = pp[c];
                 reinterpret_cast<float2*>(&sm.rc.red[1][warp][lane * CPL])[c] = rr[c];
+            }
             }
             __syncthreads();                                                           // B3
             if (tid < DV) {
@@ -639,6 +697,16 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                 S.ms[pi] = __fadd_rn(S.ms[pi], __fmul_rn(p.alpha, __fsub_rn(sm.rowR[pi], S.ms[pi])));
                 S.mr[pi] = __fadd_rn(S.mr[pi], __fmul_rn(p.alpha, __fsub_rn(xr, S.mr[pi])));
             }
+            if constexpr (RS == 2) {
+                const float2 u0 = reinterpret_cast<const float2*>(&sm.u[cl * 4])[0];
+                const float2 u1 = reinterpret_cast<const float2*>(&sm.u[cl * 4])[1];
+#pragma unroll
+                for (int jr = 0; jr < NSL; ++jr) {
+                    const float kk = kv[warp * RPW + jr * RS + half];
+                    x[jr][0] = __ffma2_rn(make_float2(kk, kk), u0, x[jr][0]);
+                    x[jr][1] = __ffma2_rn(make_float2(kk, kk), u1, x[jr][1]);
+                }
+            } else {
             float2 u2[CP2];
 #pragma unroll
             for (int c = 0; c < CP2; ++c) u2[c] = reinterpret_cast<const float2*>(&sm.u[lane * CPL])[c];
@@ -653,19 +721,17 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                     for (int c = 0; c < CP2; ++c) x[r4 + j4][c] = __ffma2_rn(k2, u2[c], x[r4 + j4][c]);
                 }
             }
+            }
         }
 
         // the payload buffer is free: the next head's packed rows
         if (has_next) wb_issue_payload<DK, DV>(sm.st[sidx ^ 1], pay, g + 1, wp);
         // state to the buffer
 #pragma unroll
-        for (int r = 0; r < RPW; ++r) {
-            const int i = warp * RPW + r;
-            if constexpr (CPL == 4)
-                *reinterpret_cast<float4*>(sm.sbuf + sb_off<DV>(i, lane)) =
-                    make_float4(x[r][0].x, x[r][0].y, x[r][1].x, x[r][1].y);
-            else
-                *reinterpret_cast<float2*>(sm.sbuf + sb_off<DV>(i, lane >> 1) + 2 * (lane & 1)) = x[r][0];
+        for (int r = 0; r < NSL; ++r) {
+            const int i = warp * RPW + r * RS + half;
+            *reinterpret_cast<float4*>(sm.sbuf + sb_off<DV>(i, cl)) =
+                make_float4(x[r][0].x, x[r][0].y, x[r][1].x, x[r][1].y);
         }
         __syncthreads();                                                               // B5
 
