@@ -25,6 +25,7 @@ import os
 import statistics
 import subprocess
 import sys
+import tempfile
 import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -109,8 +110,10 @@ class ClockSampler:
     """nvidia-smi clock / throttle sampling during the timed region."""
 
     def __init__(self, gpu_index=0):
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{gpu_index}.csv")
-        os.makedirs(os.path.dirname(self.path), exist_ok=True)
+        # raw samples go to a scratch file; the JSON line carries their summary
+        out = os.environ.get("QSTATE_CLOCKS_DIR") or tempfile.gettempdir()
+        self.path = os.path.join(out, f"qstate_clocks_rank{gpu_index}_{os.getpid()}.csv")
+        os.makedirs(out, exist_ok=True)
         self.idx = gpu_index
         self.proc = None
 
