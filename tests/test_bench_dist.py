@@ -48,3 +48,40 @@ def test_single_rank_needs_no_process_group():
     import bench
     assert bench.slowest_ms(12.5, 1, "cpu") == 12.5
     assert bench.job_throughput(500, 1, 2.0) == pytest.approx(250000.0)
+
+
+def _run_bench(args, env_extra=None):
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = dict(os.environ)
+    env.update(env_extra or {})
+    res = subprocess.run([sys.executable, os.path.join(root, "bench.py"), *args], capture_output=True,
+                         text=True, env=env, timeout=600, cwd=root)
+    return res
+
+
+def test_reference_arm_prints_the_oracle_line():
+    """`bench.py --impl reference` times the CPU oracle on host cores and prints one JSON line
+    with the bench's metric, unit and config, a cpu_baseline describing the run, and an e2e
+    block with no host-device traffic."""
+    import json
+    res = _run_bench(["--impl", "reference", "--steps", "1", "--warmup", "3", "--workload", "tiny_kda"])
+    assert res.returncode == 0, res.stderr[-2000:]
+    lines = [l for l in res.stdout.splitlines() if l.strip()]
+    assert len(lines) == 1, res.stdout
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["unit"] == "tokens/s" and d["higher_is_better"] is True
+    assert d["value"] > 0 and d["steps"] == 1 and d["warmup"] == 3
+    assert d["config"]["workload"] == "tiny_kda"
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] == 1 and cb["value"] == d["value"] and cb["sample"]
+    assert d["e2e"] == {"value": d["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}
+
+
+def test_reference_arm_other_ranks_print_nothing():
+    res = _run_bench(["--impl", "reference", "--steps", "1", "--warmup", "3", "--workload", "tiny_kda"],
+                     {"RANK": "1", "WORLD_SIZE": "2"})
+    assert res.returncode == 0, res.stderr[-2000:]
+    assert res.stdout.strip() == ""
