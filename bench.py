@@ -243,6 +243,7 @@ def config_of(w, args):
     return {"workload": w.name, "B": w.B, "H": w.H, "dk": w.dk, "dv": w.dv, "T": w.T, "C": w.C,
             "bbar": w.bbar, "widths": [w.bmin, w.bmax], "gate_bits": w.gate_bits,
             "fit_every": args.fit_every, "alloc_mode": getattr(args, "alloc_mode", 0),
+            "interval_form": getattr(args, "form", "token"),
             "global_batch": w.B * args.gpus, "seq_len": w.T,
             "parallelism": f"dp{args.gpus}",
             "l2": (f"inputs {input_gb(w):.1f} GB > 129 MB L2: no flush" if input_gb(w) > 0.129
@@ -264,6 +265,9 @@ def main():
     ap.add_argument("--fit-every", type=int, default=1)
     ap.add_argument("--alloc-mode", type=int, default=0,
                     help="0: widths from the previous write-back's statistics; 1: from this one's")
+    ap.add_argument("--form", default="token", choices=["token", "chunk"],
+                    help="write-back intervals token by token, or in 16-token blocks on the tensor "
+                         "cores (row unit, 128 x 128)")
     ap.add_argument("--T", type=int, default=None, help="tokens per step (default: workload T)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
@@ -291,7 +295,8 @@ def main():
     torch.cuda.set_device(dev)
     q.load(build_if_missing=True)
 
-    cfg = q.Config.from_workload(w, fit_every=args.fit_every, alloc_mode=args.alloc_mode)
+    cfg = q.Config.from_workload(w, fit_every=args.fit_every, alloc_mode=args.alloc_mode,
+                                 interval_form=q.FORM_CHUNK if args.form == "chunk" else q.FORM_TOKEN)
     x = synth.device_inputs(w, device=dev, seed_offset=rank_seed_offset(rank))
     nchan = w.H * w.dk
     coded = w.gate_bits > 0

@@ -60,6 +60,17 @@ extern "C" {
 #define QSTATE_ALLOC_LAGGED 0
 #define QSTATE_ALLOC_CURRENT 1
 
+/* How a write-back interval of C > 1 tokens is computed (same method, same result up to FP32
+ * rounding).  TOKEN: token by token (Eq. 1 as written).  CHUNK: in blocks of 16 tokens with
+ * the products against the block's starting state and the state update on the tensor cores
+ * (3xTF32, FP32 accumulation; Eq. 1 unrolled over the block, Sec. 2's write-back period);
+ * row unit, dk = dv = 128, erase_kind DELTA or NONE.  The chunked form needs every row's
+ * decay over a 16-token block to stay above FP32's normal range (rates summing to less than
+ * about 87 over 16 tokens); a block beyond that sets the device status (QSTATE_EDEVICE from
+ * qstate_check).  Calls whose buffers are not 16-byte aligned run the token form. */
+#define QSTATE_FORM_TOKEN 0
+#define QSTATE_FORM_CHUNK 1
+
 /* Allocation weights c_i (Eq. 3 and the alternatives of Table 1).  With the EMAs of
  * qstate_stats, m_s = EMA(1 - e^{-2s}) and m_r = EMA of the erasure term:
  * Gamma_hat = (1 - m_s) / (expm1(m_r) + m_s); Rtilde^2 = R^2 / mean of R^2 over the unit's
@@ -97,6 +108,7 @@ typedef struct qstate_cfg {
     int32_t gate_bits;           /* 0: FP32 decay rates; g in 1..8: log-quantised rates       */
     int32_t weight_kind;         /* QSTATE_WEIGHT_*                                          */
     int32_t alloc_mode;          /* QSTATE_ALLOC_LAGGED (0) or QSTATE_ALLOC_CURRENT (1)       */
+    int32_t interval_form;       /* QSTATE_FORM_TOKEN (0) or QSTATE_FORM_CHUNK (1)            */
 } qstate_cfg;
 
 /* One packed state (device pointers).  Layout (Sec. 3, "Levels and storage"; bit order is

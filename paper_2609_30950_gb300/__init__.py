@@ -17,6 +17,7 @@ QSTATE_OK, QSTATE_EINVAL, QSTATE_EBUDGET, QSTATE_ECUDA, QSTATE_EDEVICE = range(5
 DECAY_ROW, DECAY_HEAD = 0, 1
 ERASE_DELTA, ERASE_NONE, ERASE_GENERAL = 0, 1, 2
 ALLOC_LAGGED, ALLOC_CURRENT = 0, 1
+FORM_TOKEN, FORM_CHUNK = 0, 1
 UNIT_ROW, UNIT_HEAD = 0, 1
 # allocation weights (Eq. 3 and the alternatives of Table 1; see include/qstate.h)
 (WEIGHT_OURS, WEIGHT_RANGE, WEIGHT_GAMMA_RAW, WEIGHT_NRANGE, WEIGHT_PERSIST, WEIGHT_WBFACTOR,
@@ -36,7 +37,8 @@ class _Cfg(ct.Structure):
                 ("bbar_num", ct.c_int32), ("bbar_den", ct.c_int32), ("bmin", ct.c_int32),
                 ("bmax", ct.c_int32), ("C", ct.c_int32), ("fit_every", ct.c_int32),
                 ("ema_span", ct.c_float), ("gate_bits", ct.c_int32),
-                ("weight_kind", ct.c_int32), ("alloc_mode", ct.c_int32)]
+                ("weight_kind", ct.c_int32), ("alloc_mode", ct.c_int32),
+                ("interval_form", ct.c_int32)]
 
 
 class _Buf(ct.Structure):
@@ -159,6 +161,7 @@ class Config:
     gate_bits: int = 0
     weight_kind: int = 0
     alloc_mode: int = 0
+    interval_form: int = 0
 
     def c(self) -> _Cfg:
         return _Cfg(*[getattr(self, f) for f, _ in _Cfg._fields_])

@@ -14,6 +14,7 @@ cudaError_t launch_step_64x64(const qstate_cfg&, int, int, const StepParams&, cu
 cudaError_t launch_wb_row_128x128(const qstate_cfg&, const StepParams&, cudaStream_t);
 cudaError_t launch_wb_row_128x64(const qstate_cfg&, const StepParams&, cudaStream_t);
 cudaError_t launch_wb_row_64x64(const qstate_cfg&, const StepParams&, cudaStream_t);
+cudaError_t launch_wb_chunk_128x128(const qstate_cfg&, const StepParams&, cudaStream_t);
 }  // namespace qs
 
 using namespace qs;
@@ -102,6 +103,11 @@ int validate(const qstate_cfg* c) {
         return fail(QSTATE_EINVAL, "alloc_mode current is for the row unit");
     if (c->weight_kind < QSTATE_WEIGHT_OURS || c->weight_kind > QSTATE_WEIGHT_UNIFORM)
         return fail(QSTATE_EINVAL, "unsupported weight_kind %d", c->weight_kind);
+    if (c->interval_form != QSTATE_FORM_TOKEN && c->interval_form != QSTATE_FORM_CHUNK)
+        return fail(QSTATE_EINVAL, "unsupported interval_form %d", c->interval_form);
+    if (c->interval_form == QSTATE_FORM_CHUNK &&
+        (c->unit_kind != QSTATE_UNIT_ROW || c->dk != 128 || c->dv != 128 || c->erase_kind == QSTATE_ERASE_GENERAL))
+        return fail(QSTATE_EINVAL, "the chunked form needs the row unit, dk = dv = 128 and erase DELTA or NONE");
     return QSTATE_OK;
 }
 
@@ -138,6 +144,8 @@ bool wb_row_eligible(const qstate_cfg& c, const StepParams& p) {
 
 cudaError_t launch_writeback(const qstate_cfg& c, const StepParams& p, cudaStream_t st) {
     if (wb_row_eligible(c, p)) {
+        if (c.interval_form == QSTATE_FORM_CHUNK && c.dk == 128 && c.dv == 128 && !p.general)
+            return launch_wb_chunk_128x128(c, p, st);
         if (c.dk == 128 && c.dv == 128) return launch_wb_row_128x128(c, p, st);
         if (c.dk == 128 && c.dv == 64) return launch_wb_row_128x64(c, p, st);
         return launch_wb_row_64x64(c, p, st);
@@ -612,9 +620,11 @@ int qstate_check(void* stream) {
         const int zero = 0;
         e = cudaMemcpy(status, &zero, sizeof(int), cudaMemcpyHostToDevice);
         if (e != cudaSuccess) return cuda_fail(e, "status clear");
-        return fail(QSTATE_EDEVICE, "device status 0x%x:%s%s", v,
+        return fail(QSTATE_EDEVICE, "device status 0x%x:%s%s%s%s", v,
                     (v & QS_DEV_LAYOUT) ? " inconsistent widths/offsets" : "",
-                    (v & QS_DEV_RATE) ? " decay rate not positive/finite" : "");
+                    (v & QS_DEV_RATE) ? " decay rate not positive/finite" : "",
+                    (v & QS_DEV_TIMEOUT) ? " tensor-core product timed out" : "",
+                    (v & QS_DEV_CHUNK) ? " decay over a 16-token block beyond the chunked form's range" : "");
     }
     return QSTATE_OK;
 }

@@ -1,0 +1,490 @@
+// qs_chunk.cuh -- one write-back interval of a head in chunked form on the tensor cores
+// (tcgen05, sm_103a), dk = dv = 128: the row-unit write-back kernel's alternative to its
+// token-by-token loop (Eq. 1) for C > 1.
+//
+// Within a block of L = 16 tokens starting from state S_b, let d_t = e^{-s_t} (per key row),
+// Dc_t = d_0 ... d_t (decay from S_b to token t's decayed state S'_t), a_t = beta_t k_t (or 0
+// without erasure) and w_t = beta_t (or 1).  Unrolling Eq. (1) over the block gives, with
+// P(s, t) = Dc_t / Dc_s = d_{s+1} ... d_t the decay between tokens s < t:
+//     p_t = S'_t^T a_t = S_b^T (a_t o Dc_t) + sum_{s<t} A_ts u_s,   A_ts = sum_i a_ti k_si P_i(s, t)
+//     u_t = w_t v_t - p_t
+//     o_t = S_t^T q_t  = S_b^T (q_t o Dc_t) + sum_{s<=t} M_ts u_s,  M_ts = sum_i q_ti k_si P_i(s, t)
+//     S_e = Dc_{L-1} o S_b + sum_t (k_t o Dc_{L-1} / Dc_t) u_t^T.
+// The products with S_b (32 columns of S_b^T [a o Dc; q o Dc]^T), the matrices A and M (one
+// product (k / Dc) [a o Dc; q o Dc]^T) and the state update (a rank-16 product) run on the
+// tensor cores; the triangular solve for u and the readouts run on the CUDA cores.  The FP32 state stays in tensor memory (TMEM) as S^T (lane = value column j,
+// column = key row i) for the whole interval, held as its exact split S = hi + lo (hi the top
+// 19 bits, a TF32 number; lo the FP32 remainder).  The products use the 3xTF32 scheme
+// hi*hi + hi*lo + lo*hi (the tensor core truncates its inputs to TF32, so hi is exact).
+// The tensor core's FP32 accumulation truncates, so large and small terms are kept apart: the
+// hi*hi and the correction products of S_b^T [..] go to separate accumulators, and the block's
+// update goes to a fresh accumulator that the CUDA cores add to the decayed state with one
+// rounding, S_e = fma(hi + lo, Dc_{L-1}, update).
+//
+// A and M are factored as (a o Dc) . (k / Dc) over the rows: exact while every Dc of a block
+// stays a normal FP32 number, i.e. while the decay rates of one row sum to less than about 87
+// over 16 tokens; a block beyond that raises QS_DEV_CHUNK (the token-by-token kernel has no such
+// limit).
+//
+// Roles per block (256 threads): warps 0-3 own key rows (thread = row i): rates, decays, EMA
+// statistics and the operand tiles, and later value columns for the readouts; warps 4-7 stage
+// the next block's inputs and own value columns (TMEM lane j) for the solve.  All threads
+// combine and split the state.
+// Included by qs_wb_row.cuh, whose state-buffer swizzle sb_off it uses.
+#pragma once
+
+#include "qs_common.cuh"
+#include "qs_tc.cuh"
+
+namespace qs {
+
+// Defined in qs_wb_row.cuh: the state buffer's swizzle (float offset of 16-byte group G of
+// row i) and the cp.async helpers.
+template <int DV>
+__device__ __forceinline__ int sb_off(int i, int G);
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem);
+__device__ __forceinline__ void cp_async4(void* smem, const void* gmem);
+__device__ __forceinline__ void cp_async_commit();
+__device__ __forceinline__ void cp_async_wait_all();
+
+struct ChunkGeo {
+    static constexpr int L = 16;    // tokens per block
+    static constexpr int D = 128;   // dk = dv
+    // TMEM columns: S^T as hi / lo, the block's update, the product with S_b (hi*hi part and
+    // corrections), u^T hi / lo, the product (k / Dc) [a o Dc ; q o Dc]^T that gives A and M
+    static constexpr uint32_t kHi = 0, kLo = 128, kUpd = 256, kDW = 384, kDWc = 416, kUHi = 448,
+                              kULo = 464, kAM = 480;
+    static constexpr uint32_t kCols = 512;
+    // Operand tiles (K-major core matrices, see qs_tc.cuh).  A K-chunk is padded by 16 bytes
+    // where a warp writes one column of consecutive key rows, so the writes spread over all
+    // banks.
+    //  k / Dc: L rows x D (K = key row), K-chunks 272 bytes apart.  It is the A operand of an
+    //          M = 128 product: rows 16..127 alias the following bytes (always inside the
+    //          region, read but never used), their output lanes are ignored.
+    static constexpr uint32_t kLboH = L * 16 + 16, kSboH = 128;
+    //  [a o Dc ; q o Dc]: 2L rows x D, K-chunks 528 bytes apart
+    static constexpr uint32_t kLboW = 2 * L * 16 + 16, kSboW = 128;
+    //  (k o Dc_{L-1} / Dc)^T: D rows (key rows) x L (K = token)
+    static constexpr uint32_t kLboU = (D / 8) * 128, kSboU = 128;
+    static constexpr uint32_t kKh = (D / 4) * kLboH, kBw = (D / 4) * kLboW, kBu = (L / 4) * kLboU;
+    static constexpr uint32_t oKhHi = 0, oKhLo = kKh, oBwHi = 2 * kKh, oBwLo = 2 * kKh + kBw;
+    static constexpr uint32_t oBuHi = 2 * kKh + 2 * kBw, oBuLo = oBuHi + kBu;
+    static constexpr uint32_t oAM = oBuLo + kBu;                  // A and M, L x L each
+    static constexpr uint32_t oDall = oAM + 2 * L * L * 4;
+    static constexpr uint32_t oXch = oDall + D * 4;              // row preparation: the halves' exchange
+    static constexpr uint32_t oBar = oXch + 2 * D * 16;          // mbarrier (8 bytes) + TMEM address
+    // one block's token inputs, staged by cp.async one block ahead: k, q, rates (FP32 per row,
+    // per head, or uint8 codes) and beta (two buffers by block parity: the solve of block c
+    // still reads its beta when block c + 1's arrives)
+    static constexpr uint32_t oStg = oBar + 16;
+    static constexpr uint32_t sK = 0, sQ = L * D * 4, sS = 2 * L * D * 4, sB = 3 * L * D * 4;
+    static constexpr uint32_t kBytes = oStg + sB + 2 * L * 4;
+    static constexpr int kWaitPolls = 1 << 24;
+};
+static_assert(ChunkGeo::oBwHi % 16 == 0 && ChunkGeo::oBuHi % 16 == 0 && ChunkGeo::oBar % 16 == 0 &&
+              ChunkGeo::oStg % 16 == 0, "tile alignment");
+// the aliased rows of the k / Dc operand (16 row groups of 128 bytes from each K-step's start)
+// stay inside the two k / Dc tiles and the first [a o Dc ; q o Dc] tile
+static_assert(ChunkGeo::oKhLo + (ChunkGeo::D / 8 - 1) * 2 * ChunkGeo::kLboH + ChunkGeo::kLboH + 16 * 128 <=
+              ChunkGeo::oBwLo, "aliased operand rows");
+
+// Once per CTA: all 512 TMEM columns (the kernel runs one CTA per SM in this form) and the
+// mbarrier of the products.  Returns the TMEM base address.
+__device__ __forceinline__ uint32_t chunk_setup(uint8_t* cb) {
+    using G = ChunkGeo;
+    const int tid = threadIdx.x;
+    uint64_t* bar = reinterpret_cast<uint64_t*>(cb + G::oBar);
+    uint32_t* ta = reinterpret_cast<uint32_t*>(cb + G::oBar + 8);
+    if (tid < 32) {
+        tc::tmem_alloc(ta, G::kCols);
+        tc::tmem_relinquish();
+    }
+    if (tid == 32) {
+        tc::mbar_init(bar, 1);
+        tc::mbar_fence_init();
+    }
+    tc::fence_before_sync();
+    __syncthreads();
+    tc::fence_after_sync();
+    return *ta;
+}
+
+__device__ __forceinline__ void chunk_teardown(uint32_t tmem) {
+    tc::fence_before_sync();
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        tc::fence_after_sync();
+        tc::tmem_dealloc(tmem, ChunkGeo::kCols);
+    }
+}
+
+// The interval [p.t_begin, p.t_end) of head (b, h): the state arrives in sbuf (row-major,
+// swizzled) and leaves there; readouts go to p.o, the EMA statistics of the rows to S.ms / S.mr.
+// `phase` tracks the mbarrier's parity (uniform over the CTA).
+template <class Stage>
+__device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, float* sbuf, uint8_t* cb,
+                                               uint32_t tmem, uint32_t& phase, int b, int h, bool stats) {
+    using G = ChunkGeo;
+    constexpr int L = G::L, D = G::D;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int sub = warp & 3, hf = warp >> 2;
+    const int jl = 32 * sub + lane;   // the TMEM lane (value column) this thread addresses
+    const int tt = tid - 128;         // index among the value-column threads (warps 4-7)
+    const uint32_t tl = tmem + (static_cast<uint32_t>(32 * sub) << 16);
+    uint64_t* bar = reinterpret_cast<uint64_t*>(cb + G::oBar);
+    float* amA = reinterpret_cast<float*>(cb + G::oAM);
+    float* amM = amA + L * L;
+    float* dall = reinterpret_cast<float*>(cb + G::oDall);
+    uint8_t* kh_hi = cb + G::oKhHi;
+    uint8_t* kh_lo = cb + G::oKhLo;
+    uint8_t* bw_hi = cb + G::oBwHi;
+    uint8_t* bw_lo = cb + G::oBwLo;
+    uint8_t* bu_hi = cb + G::oBuHi;
+    uint8_t* bu_lo = cb + G::oBuLo;
+    uint8_t* stg = cb + G::oStg;
+    const float* sk = reinterpret_cast<const float*>(stg + G::sK);
+    const float* sq = reinterpret_cast<const float*>(stg + G::sQ);
+    const float* ss = reinterpret_cast<const float*>(stg + G::sS);
+    const uint8_t* sc = stg + G::sS;
+    const size_t tokb = static_cast<size_t>(b) * p.T;
+    auto wait_mma = [&]() {
+        if (!tc::mbar_wait(bar, phase, G::kWaitPolls)) raise_status(p.status, QS_DEV_TIMEOUT);
+        phase ^= 1u;
+        tc::fence_after_sync();
+    };
+    // staging of the block at token tb by the value-column threads: k, q, the rates and beta
+    auto issue_kqs = [&](int tb) {
+        const int nb = min(L, p.t_end - tb);
+        if (p.erase && tt < nb)
+            cp_async4(stg + G::sB + (((tb - p.t_begin) / L) & 1) * L * 4 + tt * 4, p.beta + (tokb + tb + tt) * p.H + h);
+        for (int c = tt; c < nb * (D / 4); c += 128) {
+            const int tau = c / (D / 4), part = c % (D / 4);
+            const size_t tok = (tokb + tb + tau) * p.H + h;
+            cp_async16(stg + G::sK + tau * D * 4 + part * 16, p.k + tok * D + part * 4);
+            cp_async16(stg + G::sQ + tau * D * 4 + part * 16, p.q + tok * D + part * 4);
+            if (p.decay_row && !p.s_code) cp_async16(stg + G::sS + tau * D * 4 + part * 16, p.s + tok * D + part * 4);
+        }
+        if (p.decay_row && p.s_code) {
+            for (int c = tt; c < nb * (D / 16); c += 128) {
+                const int tau = c / (D / 16), part = c % (D / 16);
+                const size_t tok = (tokb + tb + tau) * p.H + h;
+                cp_async16(stg + G::sS + tau * D + part * 16, p.s_code + tok * D + part * 16);
+            }
+        } else if (!p.decay_row && tt < nb) {
+            const size_t tok = (tokb + tb + tt) * p.H + h;
+            if (p.s_code)   // one code per head and token: its level, stored directly
+                reinterpret_cast<float*>(stg + G::sS)[tt] =
+                    __ldg(p.s_lut + static_cast<size_t>(h) * p.L + min(static_cast<int>(p.s_code[tok]), p.L - 1));
+            else
+                cp_async4(stg + G::sS + tt * 4, p.s + tok);
+        }
+        cp_async_commit();
+    };
+    if (tt >= 0 && p.t_begin < p.t_end) issue_kqs(p.t_begin);
+
+    // state in: S^T into TMEM as hi / lo; this thread's lane j, key rows of its half
+#pragma unroll 1
+    for (int i0 = 64 * hf; i0 < 64 * hf + 64; i0 += 16) {
+        float hi[16], lo[16];
+#pragma unroll
+        for (int c = 0; c < 16; ++c) {
+            const float x = sbuf[sb_off<D>(i0 + c, jl >> 2) + (jl & 3)];
+            hi[c] = tc::tf32_hi(x);
+            lo[c] = __fsub_rn(x, hi[c]);
+        }
+        tc::tmem_st16(tl + G::kHi + i0, hi);
+        tc::tmem_st16(tl + G::kLo + i0, lo);
+    }
+    tc::wait_st();
+    tc::fence_before_sync();
+
+#pragma unroll 1
+    for (int t0 = p.t_begin; t0 < p.t_end; t0 += L) {
+        const int n = min(L, p.t_end - t0);
+        const bool last = t0 + L >= p.t_end;
+        const float* sbeta = reinterpret_cast<const float*>(stg + G::sB) + (((t0 - p.t_begin) / L) & 1) * L;
+        // this block's k, q, rates and beta have landed
+        if (tt >= 0) cp_async_wait_all();
+        __syncthreads();                                                            // C0
+        float vv[L];
+        if (hf == 1) {
+            // value-column role: this block's v, in flight while the rows are prepared
+#pragma unroll
+            for (int t = 0; t < L; ++t)
+                vv[t] = t < n ? __ldg(p.v + ((tokb + t0 + t) * p.H + h) * D + jl) : 0.0f;
+        }
+        // Rows: thread (i, half hh) takes tokens 8 hh .. 8 hh + 7 of key row i.  The halves
+        // exchange through shared memory the first half's decay product and EMA state (for
+        // the second) and the second half's decay product (for the first half's end-of-block
+        // factors); the EMA recursion runs token by token in order.
+        constexpr int LH = L / 2;
+        const int i = tid & (D - 1), hh = tid >> 7, tb = LH * hh;
+        float4* xch = reinterpret_cast<float4*>(cb + G::oXch);
+        float kk[LH], dd[LH], pr[LH], sf[LH];
+        {
+            float xs[LH], xr[LH], qv[LH], bv[LH];
+#pragma unroll
+            for (int j = 0; j < LH; ++j) {
+                const int tau = tb + j;
+                kk[j] = qv[j] = bv[j] = xs[j] = xr[j] = 0.0f;
+                dd[j] = 1.0f;
+                if (tau < n) {
+                    kk[j] = sk[tau * D + i];
+                    qv[j] = sq[tau * D + i];
+                    if (p.erase) bv[j] = sbeta[tau];
+                    float rate;
+                    if (!p.decay_row) {
+                        rate = ss[tau];
+                    } else if (p.s_code) {
+                        const int code = min(static_cast<int>(sc[tau * D + i]), p.L - 1);
+                        rate = p.L <= 4 ? S.lut[i * p.L + code]
+                                        : __ldg(p.s_lut + (static_cast<size_t>(h) * D + i) * p.L + code);
+                    } else {
+                        rate = ss[tau * D + i];
+                    }
+                    if (!(rate > 0.0f) || !(rate < INFINITY)) raise_status(p.status, QS_DEV_RATE);
+                    dd[j] = expf(-rate);
+                    if (stats) {
+                        xs[j] = -expm1f(-2.0f * rate);
+                        xr[j] = p.erase ? __fmul_rn(__fmul_rn(bv[j], __fsub_rn(2.0f, bv[j])), __fmul_rn(kk[j], kk[j])) : 0.0f;
+                    }
+                }
+            }
+            // decay products within the half: pr[j] = d_tb ... d_{tb+j}, sf[j] = d_{tb+j+1} ... d_{tb+LH-1}
+            float acc = 1.0f;
+#pragma unroll
+            for (int j = 0; j < LH; ++j) pr[j] = acc = __fmul_rn(acc, dd[j]);
+            acc = 1.0f;
+#pragma unroll
+            for (int j = LH - 1; j >= 0; --j) {
+                sf[j] = acc;
+                acc = __fmul_rn(acc, dd[j]);
+            }
+            if (hh == 0) {
+                float ms = stats ? S.ms[i] : 0.0f, mr = stats ? S.mr[i] : 0.0f;
+                if (stats) {
+#pragma unroll
+                    for (int j = 0; j < LH; ++j) {
+                        if (j >= n) break;
+                        if (t0 + j == 0) {
+                            ms = xs[j];
+                            mr = xr[j];
+                        } else {
+                            ms = __fadd_rn(ms, __fmul_rn(p.alpha, __fsub_rn(xs[j], ms)));
+                            mr = __fadd_rn(mr, __fmul_rn(p.alpha, __fsub_rn(xr[j], mr)));
+                        }
+                    }
+                }
+                xch[i] = make_float4(pr[LH - 1], ms, mr, 0.0f);
+            } else {
+                xch[D + i].x = pr[LH - 1];
+            }
+            __syncthreads();                                                        // Cx
+            const float4 x0 = xch[i];
+            const float dc0 = hh == 0 ? 1.0f : x0.x;            // decay before the half
+            const float sf1 = hh == 0 ? xch[D + i].x : 1.0f;   // decay after the half, in the block
+            if (hh == 1) {
+                // the EMA state after the whole block and the block's decay (with no second-half
+                // tokens, the first half's)
+                float ms = x0.y, mr = x0.z;
+                if (stats) {
+#pragma unroll
+                    for (int j = 0; j < LH; ++j) {
+                        if (tb + j >= n) break;
+                        ms = __fadd_rn(ms, __fmul_rn(p.alpha, __fsub_rn(xs[j], ms)));
+                        mr = __fadd_rn(mr, __fmul_rn(p.alpha, __fsub_rn(xr[j], mr)));
+                    }
+                    S.ms[i] = ms;
+                    S.mr[i] = mr;
+                }
+                const float Dall = __fmul_rn(dc0, pr[LH - 1]);
+                if (!(Dall >= 1e-37f)) raise_status(p.status, QS_DEV_CHUNK);
+                dall[i] = Dall;
+            }
+            const int oh = (i >> 2) * G::kLboH + (i & 3) * 4, ow = (i >> 2) * G::kLboW + (i & 3) * 4;
+#pragma unroll
+            for (int j = 0; j < LH; ++j) {
+                const int tau = tb + j;
+                const float Dc = __fmul_rn(dc0, pr[j]);
+                const float a = p.erase ? __fmul_rn(bv[j], kk[j]) : 0.0f;
+                const float kt = __fmul_rn(a, Dc), qt = __fmul_rn(qv[j], Dc);
+                float rDc;   // k / Dc only enters A and M
+                asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(rDc) : "f"(Dc));
+                const float kh = tau < n ? __fmul_rn(kk[j], rDc) : 0.0f;
+                // tiles: k / Dc row tau; [a o Dc ; q o Dc] rows tau and L + tau (row r of a
+                // K-chunk at byte 16 r)
+                const float khh = tc::tf32_hi(kh), kth = tc::tf32_hi(kt), qth = tc::tf32_hi(qt);
+                *reinterpret_cast<float*>(kh_hi + oh + 16 * tau) = khh;
+                *reinterpret_cast<float*>(kh_lo + oh + 16 * tau) = __fsub_rn(kh, khh);
+                *reinterpret_cast<float*>(bw_hi + ow + 16 * tau) = kth;
+                *reinterpret_cast<float*>(bw_lo + ow + 16 * tau) = __fsub_rn(kt, kth);
+                *reinterpret_cast<float*>(bw_hi + ow + 16 * (L + tau)) = qth;
+                *reinterpret_cast<float*>(bw_lo + ow + 16 * (L + tau)) = __fsub_rn(qt, qth);
+            }
+            // (k o Dc_{L-1} / Dc)^T: row i, tokens of the half, 4 per 16-byte chunk
+#pragma unroll
+            for (int c4 = 0; c4 < LH / 4; ++c4) {
+                float kb[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) kb[e] = __fmul_rn(kk[4 * c4 + e], __fmul_rn(sf[4 * c4 + e], sf1));
+                float4 hi, lo;
+                hi.x = tc::tf32_hi(kb[0]);
+                hi.y = tc::tf32_hi(kb[1]);
+                hi.z = tc::tf32_hi(kb[2]);
+                hi.w = tc::tf32_hi(kb[3]);
+                lo.x = __fsub_rn(kb[0], hi.x);
+                lo.y = __fsub_rn(kb[1], hi.y);
+                lo.z = __fsub_rn(kb[2], hi.z);
+                lo.w = __fsub_rn(kb[3], hi.w);
+                const int o = ((tb >> 2) + c4) * G::kLboU + (i >> 3) * G::kSboU + (i & 7) * 16;
+                *reinterpret_cast<float4*>(bu_hi + o) = hi;
+                *reinterpret_cast<float4*>(bu_lo + o) = lo;
+            }
+        }
+        tc::fence_async_smem();
+        __syncthreads();                                                            // C1
+
+        // On the tensor cores (3xTF32, K = 128 key rows): S_b^T [a o Dc ; q o Dc]^T, its hi*hi
+        // product and the two corrections in separate accumulators, and (k / Dc) [a o Dc ;
+        // q o Dc]^T, whose row s, column t is A_ts (column < L) or M_ts (column >= L)
+        if (tid == 0) {
+            tc::fence_after_sync();
+            constexpr uint32_t idW = tc::idesc_tf32(128, 2 * L);
+            // a K-step advances the start addresses (16-byte units, bits 0-13) by two K-chunks
+            constexpr uint64_t kStepW = (2 * G::kLboW) >> 4, kStepH = (2 * G::kLboH) >> 4;
+            uint64_t bh = tc::smem_desc(tc::smem_addr(bw_hi), G::kLboW, G::kSboW);
+            uint64_t bl = tc::smem_desc(tc::smem_addr(bw_lo), G::kLboW, G::kSboW);
+            uint64_t ah = tc::smem_desc(tc::smem_addr(kh_hi), G::kLboH, G::kSboH);
+            uint64_t al = tc::smem_desc(tc::smem_addr(kh_lo), G::kLboH, G::kSboH);
+#pragma unroll
+            for (int ks = 0; ks < D / 8; ++ks) {
+                const uint32_t acc = ks > 0 ? 1u : 0u;
+                tc::mma_tf32_ts(tmem + G::kDW, tmem + G::kHi + 8 * ks, bh, idW, acc);
+                tc::mma_tf32_ts(tmem + G::kDWc, tmem + G::kHi + 8 * ks, bl, idW, acc);
+                tc::mma_tf32_ts(tmem + G::kDWc, tmem + G::kLo + 8 * ks, bh, idW, 1u);
+                tc::mma_tf32_ss(tmem + G::kAM, ah, bh, idW, acc);
+                tc::mma_tf32_ss(tmem + G::kAM, ah, bl, idW, 1u);
+                tc::mma_tf32_ss(tmem + G::kAM, al, bh, idW, 1u);
+                bh += kStepW;
+                bl += kStepW;
+                ah += kStepH;
+                al += kStepH;
+            }
+            tc::mma_commit(bar);
+        }
+        // the rows are prepared: the next block's k, q, rates and beta can come in
+        if (tt >= 0 && !last) issue_kqs(t0 + L);
+        wait_mma();
+        if (warp == 0) {
+            // A and M to shared memory (lane s < L holds row s of the product)
+            float x[L], y[L];
+            tc::tmem_ld2x16(tl + G::kAM, tl + G::kAM + L, x, y);
+            if (lane < L) {
+#pragma unroll
+                for (int t = 0; t < L; ++t) {
+                    amA[t * L + lane] = x[t];
+                    amM[t * L + lane] = y[t];
+                }
+            }
+        }
+        __syncthreads();                                                            // C2
+
+        if (hf == 1) {
+            // u of column j, token by token: u_t = w_t v_t - (S_b^T (a o Dc))_t - sum_{s<t} A_ts u_s
+            float wk[L], ck[L];
+            tc::tmem_ld2x16(tl + G::kDW, tl + G::kDWc, wk, ck);
+            float u[L];
+#pragma unroll
+            for (int t = 0; t < L; ++t) {
+                float pp = __fadd_rn(wk[t], ck[t]);
+#pragma unroll
+                for (int s = 0; s < t; ++s) pp = fmaf(amA[t * L + s], u[s], pp);
+                const float bt = p.erase ? sbeta[t] : 1.0f;
+                u[t] = t < n ? (p.erase ? __fsub_rn(__fmul_rn(bt, vv[t]), pp) : vv[t]) : 0.0f;
+            }
+            float uh[L], ul[L];
+#pragma unroll
+            for (int t = 0; t < L; ++t) {
+                uh[t] = tc::tf32_hi(u[t]);
+                ul[t] = __fsub_rn(u[t], uh[t]);
+            }
+            tc::tmem_st16(tl + G::kUHi, uh);
+            tc::tmem_st16(tl + G::kULo, ul);
+            tc::wait_st();
+        }
+        tc::fence_before_sync();
+        __syncthreads();                                                            // C3
+
+        // update = u^T (k o Dc_{L-1} / Dc) on the tensor cores (3xTF32, K = 16 tokens)
+        if (tid == 0) {
+            tc::fence_after_sync();
+            constexpr uint32_t idU = tc::idesc_tf32(128, D);
+            constexpr uint64_t kStepU = (2 * G::kLboU) >> 4;
+            uint64_t bh = tc::smem_desc(tc::smem_addr(bu_hi), G::kLboU, G::kSboU);
+            uint64_t bl = tc::smem_desc(tc::smem_addr(bu_lo), G::kLboU, G::kSboU);
+#pragma unroll
+            for (int ks = 0; ks < L / 8; ++ks) {
+                tc::mma_tf32_ts(tmem + G::kUpd, tmem + G::kUHi + 8 * ks, bh, idU, ks > 0 ? 1u : 0u);
+                tc::mma_tf32_ts(tmem + G::kUpd, tmem + G::kUHi + 8 * ks, bl, idU, 1u);
+                tc::mma_tf32_ts(tmem + G::kUpd, tmem + G::kULo + 8 * ks, bh, idU, 1u);
+                bh += kStepU;
+                bl += kStepU;
+            }
+            tc::mma_commit(bar);
+        }
+        if (hf == 0) {
+            // readouts of column j: o_t = (S_b^T (q o Dc))_t + sum_{s<=t} M_ts u_s, with u from
+            // its hi / lo parts in TMEM (written by the value-column thread of the same lane)
+            float wq[L], cq[L], uh[L], ul[L];
+            tc::tmem_ld2x16(tl + G::kDW + L, tl + G::kDWc + L, wq, cq);
+            tc::tmem_ld2x16(tl + G::kUHi, tl + G::kULo, uh, ul);
+#pragma unroll
+            for (int t = 0; t < L; ++t) {
+                float oa = __fadd_rn(wq[t], cq[t]), ob = 0.0f;
+#pragma unroll
+                for (int s = 0; s <= t; s += 2) {
+                    oa = fmaf(amM[t * L + s], __fadd_rn(uh[s], ul[s]), oa);
+                    if (s + 1 <= t) ob = fmaf(amM[t * L + s + 1], __fadd_rn(uh[s + 1], ul[s + 1]), ob);
+                }
+                if (t < n) p.o[((tokb + t0 + t) * p.H + h) * D + jl] = oa + ob;
+            }
+        }
+        wait_mma();
+        // S_e = fma(hi + lo, Dc_{L-1}, update): to hi / lo for the next block, or, after the
+        // interval's last block, to the row-major buffer
+#pragma unroll 1
+        for (int c0 = 64 * hf; c0 < 64 * hf + 64; c0 += 16) {
+            float hi[16], lo[16], up[16];
+            tc::tmem_ld2x16(tl + G::kHi + c0, tl + G::kLo + c0, hi, lo);
+            tc::tmem_ld16(tl + G::kUpd + c0, up);
+#pragma unroll
+            for (int c = 0; c < 16; ++c) {
+                const float x = fmaf(__fadd_rn(hi[c], lo[c]), dall[c0 + c], up[c]);
+                if (last) {
+                    sbuf[sb_off<D>(c0 + c, jl >> 2) + (jl & 3)] = x;
+                } else {
+                    hi[c] = tc::tf32_hi(x);
+                    lo[c] = __fsub_rn(x, hi[c]);
+                }
+            }
+            if (!last) {
+                tc::tmem_st16(tl + G::kHi + c0, hi);
+                tc::tmem_st16(tl + G::kLo + c0, lo);
+            }
+        }
+        if (!last) tc::wait_st();
+        tc::fence_before_sync();
+    }
+    if (p.t_begin >= p.t_end) {
+        // no tokens: the state goes back unchanged
+#pragma unroll 1
+        for (int i0 = 64 * hf; i0 < 64 * hf + 64; i0 += 16) {
+            float hi[16], lo[16];
+            tc::tmem_ld2x16(tl + G::kHi + i0, tl + G::kLo + i0, hi, lo);
+#pragma unroll
+            for (int c = 0; c < 16; ++c) sbuf[sb_off<D>(i0 + c, jl >> 2) + (jl & 3)] = __fadd_rn(hi[c], lo[c]);
+        }
+    }
+}
+
+}  // namespace qs

@@ -12,6 +12,8 @@ namespace qs {
 enum : int {
     QS_DEV_LAYOUT = 1,  // widths/offsets inconsistent with the region
     QS_DEV_RATE = 2,    // a decay rate is not a positive finite number
+    QS_DEV_TIMEOUT = 4, // a tensor-core product did not signal completion in time
+    QS_DEV_CHUNK = 8,   // chunked form: a row's decay over a 16-token block leaves FP32 range
 };
 
 constexpr int kNFit = 16;

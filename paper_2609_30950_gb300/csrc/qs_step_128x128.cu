@@ -10,4 +10,7 @@ cudaError_t launch_step_128x128(const qstate_cfg& cfg, int src_packed, int dst_p
 cudaError_t launch_wb_row_128x128(const qstate_cfg& cfg, const StepParams& p, cudaStream_t stream) {
     return launch_wb_row_t<128, 128, 8>(cfg, p, stream);
 }
+cudaError_t launch_wb_chunk_128x128(const qstate_cfg& cfg, const StepParams& p, cudaStream_t stream) {
+    return launch_wb_row_t<128, 128, 8, true>(cfg, p, stream);
+}
 }  // namespace qs

@@ -43,6 +43,7 @@
 #include <algorithm>
 
 #include "qs_common.cuh"
+#include "qs_chunk.cuh"   // the chunked form of the interval
 
 namespace qs {
 
@@ -300,8 +301,10 @@ __device__ __forceinline__ void wb_issue_payload(const WbStage<DK, DV>& S, uint8
 }
 
 // ---- the kernel ---------------------------------------------------------------------------------
-template <int DK, int DV, int NW>
-__global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
+// CHUNK: the interval runs in chunked form on the tensor cores (qs_chunk.cuh; dk = dv = 128),
+// one CTA per SM (all of TMEM, about 190 KB of shared memory); otherwise token by token.
+template <int DK, int DV, int NW, bool CHUNK = false>
+__global__ void __launch_bounds__(NW * 32, CHUNK ? 1 : 2) wb_row_kernel(const WbParams wp) {
     using Geo = WbGeom<DK, DV, NW>;
     constexpr int RPW = Geo::RPW, CPL = Geo::CPL, CP2 = CPL / 2;
     constexpr int TPR = Geo::TPR, RPB = Geo::RPB, KPT = Geo::KPT, NB = DK / RPB;
@@ -328,6 +331,9 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
     const int g_begin = static_cast<int>(static_cast<long long>(blockIdx.x) * wp.nheads / gridDim.x);
     const int g_end = static_cast<int>(static_cast<long long>(blockIdx.x + 1) * wp.nheads / gridDim.x);
     if (g_begin >= g_end) return;
+    uint8_t* cb = pay + ((p.stage_bytes + 32 + 15) & ~15);   // chunked form's region
+    uint32_t tmem = 0, mphase = 0;
+    if constexpr (CHUNK) tmem = chunk_setup(cb);
     {
         const int h0 = g_begin % p.H;
         const int io = static_cast<int>(p.in_head_off[g_begin]);
@@ -408,9 +414,9 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                 }
             }
             if (!(rate > 0.0f) || !(rate < INFINITY)) raise_status(p.status, QS_DEV_RATE);
-            const float d = expf(-rate);
+            const float d = CHUNK ? 1.0f : expf(-rate);   // the chunked form decays every token itself
             const float ai = p.general ? S.ga[i] : __fmul_rn(beta0, kk);
-            if (stats) {
+            if (stats && !CHUNK) {
                 const float xs = -expm1f(-2.0f * rate);
                 float xr = p.erase ? __fmul_rn(__fmul_rn(beta0, __fsub_rn(2.0f, beta0)), __fmul_rn(kk, kk)) : 0.0f;
                 if (p.general) xr = general_erasure<DK>(ai, kk, S.k);
@@ -548,8 +554,8 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
                 if (p.general) rw = __ldg(p.w_in + tn * DV + pi);
             }
         };
-        if (prep_k && p.t_begin + 1 < p.t_end) load_raw(tok0 + p.H);
-        for (int t = p.t_begin, j = 0; t < p.t_end; ++t, ++j) {
+        if (!CHUNK && prep_k && p.t_begin + 1 < p.t_end) load_raw(tok0 + p.H);
+        for (int t = p.t_begin, j = 0; !CHUNK && t < p.t_end; ++t, ++j) {
             const size_t tok = (static_cast<size_t>(b) * T + t) * p.H + h;
             const int cb = j & 1, k3 = j % 3;
             const float* kv = k3 == 0 ? S.k : k3 == 1 ? sm.tk : sm.tk2;
@@ -733,6 +739,10 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
             *reinterpret_cast<float4*>(sm.sbuf + sb_off<DV>(i, cl)) =
                 make_float4(x[r][0].x, x[r][0].y, x[r][1].x, x[r][1].y);
         }
+        if constexpr (CHUNK) {
+            __syncthreads();
+            chunk_interval(p, S, sm.sbuf, cb, tmem, mphase, b, h, stats);
+        }
         __syncthreads();                                                               // B5
 
         // ---- write-back (row layout) ----------------------------------------------------------
@@ -894,17 +904,18 @@ __global__ void __launch_bounds__(NW * 32, 2) wb_row_kernel(const WbParams wp) {
             }
         }
     }
+    if constexpr (CHUNK) chunk_teardown(tmem);
 }
 
-template <int DK, int DV, int NW>
+template <int DK, int DV, int NW, bool CHUNK = false>
 cudaError_t launch_wb_row_t(const qstate_cfg& cfg, const StepParams& sp, cudaStream_t stream) {
-    auto kern = wb_row_kernel<DK, DV, NW>;
+    auto kern = wb_row_kernel<DK, DV, NW, CHUNK>;
     WbParams wp;
     wp.s = sp;
     wp.s.stage_bytes = DK * DV * cfg.bmax / 8;
     wp.nheads = cfg.B * cfg.H;
     const int pstride = (wp.s.stage_bytes + 32 + 15) & ~15;
-    const size_t smem = sizeof(WbSmem<DK, DV, NW>) + static_cast<size_t>(pstride);
+    const size_t smem = sizeof(WbSmem<DK, DV, NW>) + static_cast<size_t>(pstride) + (CHUNK ? ChunkGeo::kBytes : 0u);
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;

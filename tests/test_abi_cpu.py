@@ -72,3 +72,19 @@ def test_calls_reject_null_pointers_without_launching(lib):
     cfg = q.Config(B=1, H=1, dk=64, dv=64, bbar_num=2, bmin=1, bmax=16).c()
     assert lib.qstate_pack(ct.byref(cfg), None, None, None, None) == q.QSTATE_EINVAL
     assert b"null" in lib.qstate_last_error()
+
+
+def test_chunked_form_configuration_limits(lib):
+    """The chunked form (interval_form = 1) is for the row unit at dk = dv = 128 with the
+    delta rule or no erasure; anything else is rejected before a launch."""
+    import paper_2609_30950_gb300 as q
+    q.validate(q.Config(B=1, H=2, dk=128, dv=128, interval_form=q.FORM_CHUNK))
+    q.validate(q.Config(B=1, H=2, dk=128, dv=128, erase_kind=q.ERASE_NONE, decay_kind=q.DECAY_HEAD,
+                        interval_form=q.FORM_CHUNK))
+    for kw in (dict(dk=64, dv=64), dict(unit_kind=q.UNIT_HEAD, decay_kind=q.DECAY_HEAD),
+               dict(erase_kind=q.ERASE_GENERAL), dict(interval_form=2)):
+        base = dict(B=1, H=2, dk=128, dv=128, interval_form=q.FORM_CHUNK)
+        base.update(kw)
+        with pytest.raises(q.QstateError) as e:
+            q.validate(q.Config(**base))
+        assert e.value.code == q.QSTATE_EINVAL

@@ -219,12 +219,16 @@ def test_fp32_recurrence_free_running(qs, orc, name):
 
 
 # --------------------------------------------------------------- quantised write-backs, lockstep
-def _lockstep(qs, orc, w, fit_every=1, log_decay=False, sample_b=None, max_wb=None, weight_kind=0):
+def _lockstep(qs, orc, w, fit_every=1, log_decay=False, sample_b=None, max_wb=None, weight_kind=0,
+              interval_form=0):
     """Run the oracle free; before every write-back copy its state into the GPU, run one
     qstate_step and compare the GPU's write-back with the oracle's.  With sample_b, the GPU
     runs the full batch and only those batch elements are injected and compared (the oracle
-    runs a B=1 configuration per sampled element)."""
-    cfgq = qs.Config.from_workload(w, fit_every=fit_every, weight_kind=weight_kind)
+    runs a B=1 configuration per sampled element).  interval_form selects the library's
+    token-by-token or chunked computation of each interval (the oracle is always token by
+    token)."""
+    cfgq = qs.Config.from_workload(w, fit_every=fit_every, weight_kind=weight_kind,
+                                   interval_form=interval_form)
     cfgo_full = orc.Cfg.from_workload(w, fit_every=fit_every, weight_kind=weight_kind)
     inp = synth.host_inputs(w)
     s_code = s_lut = None
@@ -292,9 +296,9 @@ def _lockstep(qs, orc, w, fit_every=1, log_decay=False, sample_b=None, max_wb=No
                              g_out.fidx[key * groups:(key + 1) * groups])
             else:
                 gb = g_out
-            st = compare_packed(orc, cfgo, gb, S["dst"], X=xo)
-            # statistics
             us = slice(key * units, (key + 1) * units) if one else slice(None)
+            st = compare_packed(orc, cfgo, gb, S["dst"], X=xo, R_gpu=g_R[us], R_ref=S["R"])
+            # statistics
             for a, r in ((g_ms[us], S["ms"]), (g_mr[us], S["mr"])):
                 assert np.allclose(a, r, rtol=REL_STATS, atol=1e-30), wi
             if cfgo.unit_kind == 0:

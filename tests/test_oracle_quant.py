@@ -206,3 +206,17 @@ def test_log_decay_degenerate_and_invalid(orc):
     assert np.all(lut == np.float32(0.2)) and np.all(codes == 3)
     with pytest.raises(ValueError):
         orc.quant_decay(np.zeros((4, 2), np.float32), 2, 2)
+
+
+def test_parity_candidate_errors_match_the_oracle(orc):
+    """The parity helper that rebuilds a group's candidate errors from a given range
+    (used where GPU and oracle ranges round one candidate step to neighbouring FP16 numbers)
+    gives the oracle's own candidate errors when handed the group's own range."""
+    from parity import candidate_sse
+    rng = np.random.default_rng(11)
+    for b in (2, 3, 4, 6, 8, 12, 16):
+        for _ in range(6):
+            x = (rng.standard_normal(128) * np.exp(rng.normal(0, 2))).astype(np.float32)
+            _, _, _, sse = orc.quant_group(x, b, with_sse=True)
+            got = candidate_sse(x, b, np.max(np.abs(x)))
+            assert np.allclose(got, sse, rtol=1e-12, atol=0), (b, got, sse)
