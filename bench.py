@@ -265,9 +265,9 @@ def main():
     ap.add_argument("--fit-every", type=int, default=1)
     ap.add_argument("--alloc-mode", type=int, default=0,
                     help="0: widths from the previous write-back's statistics; 1: from this one's")
-    ap.add_argument("--form", default="token", choices=["token", "chunk"],
+    ap.add_argument("--form", default="auto", choices=["auto", "token", "chunk"],
                     help="write-back intervals token by token, or in 16-token blocks on the tensor "
-                         "cores (row unit, 128 x 128)")
+                         "cores (row unit, 128 x 128, C > 1); auto: the chunked form where it applies")
     ap.add_argument("--T", type=int, default=None, help="tokens per step (default: workload T)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
@@ -295,6 +295,9 @@ def main():
     torch.cuda.set_device(dev)
     q.load(build_if_missing=True)
 
+    if args.form == "auto":
+        args.form = ("chunk" if w.C > 1 and w.unit == "row" and w.dk == 128 and w.dv == 128
+                     and not w.general else "token")
     cfg = q.Config.from_workload(w, fit_every=args.fit_every, alloc_mode=args.alloc_mode,
                                  interval_form=q.FORM_CHUNK if args.form == "chunk" else q.FORM_TOKEN)
     x = synth.device_inputs(w, device=dev, seed_offset=rank_seed_offset(rank))

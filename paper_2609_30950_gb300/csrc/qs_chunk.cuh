@@ -46,6 +46,11 @@ __device__ __forceinline__ void cp_async16(void* smem, const void* gmem);
 __device__ __forceinline__ void cp_async4(void* smem, const void* gmem);
 __device__ __forceinline__ void cp_async_commit();
 __device__ __forceinline__ void cp_async_wait_all();
+// Wait until at most N of this thread's cp.async groups are pending (groups complete in order).
+template <int N>
+__device__ __forceinline__ void cp_async_wait_group() {
+    asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+}
 
 struct ChunkGeo {
     static constexpr int L = 16;    // tokens per block
@@ -59,7 +64,7 @@ struct ChunkGeo {
     // where a warp writes one column of consecutive key rows, so the writes spread over all
     // banks.
     //  k / Dc: L rows x D (K = key row), K-chunks 272 bytes apart.  It is the A operand of an
-    //          M = 128 product: rows 16..127 alias the following bytes (always inside the
+    //          M = 64 product: rows 16..63 alias the following bytes (always inside the
     //          region, read but never used), their output lanes are ignored.
     static constexpr uint32_t kLboH = L * 16 + 16, kSboH = 128;
     //  [a o Dc ; q o Dc]: 2L rows x D, K-chunks 528 bytes apart
@@ -180,6 +185,16 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
         }
         cp_async_commit();
     };
+    // ... and v, into the row-major state buffer, which is free between the state's way in and
+    // the last block's way out (global loads in flight would hold up every barrier)
+    auto issue_v = [&](int tb) {
+        const int nb = min(L, p.t_end - tb);
+        for (int c = tt; c < nb * (D / 4); c += 128) {
+            const int tau = c / (D / 4), part = c % (D / 4);
+            cp_async16(sbuf + tau * D + part * 4, p.v + ((tokb + tb + tau) * p.H + h) * D + part * 4);
+        }
+        cp_async_commit();
+    };
     if (tt >= 0 && p.t_begin < p.t_end) issue_kqs(p.t_begin);
 
     // state in: S^T into TMEM as hi / lo; this thread's lane j, key rows of its half
@@ -203,16 +218,15 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
         const int n = min(L, p.t_end - t0);
         const bool last = t0 + L >= p.t_end;
         const float* sbeta = reinterpret_cast<const float*>(stg + G::sB) + (((t0 - p.t_begin) / L) & 1) * L;
-        // this block's k, q, rates and beta have landed
-        if (tt >= 0) cp_async_wait_all();
-        __syncthreads();                                                            // C0
-        float vv[L];
-        if (hf == 1) {
-            // value-column role: this block's v, in flight while the rows are prepared
-#pragma unroll
-            for (int t = 0; t < L; ++t)
-                vv[t] = t < n ? __ldg(p.v + ((tokb + t0 + t) * p.H + h) * D + jl) : 0.0f;
+        // this block's k, q, rates and beta have landed (the first block's v is not yet asked for;
+        // a later block's may still be in flight)
+        const bool first = t0 == p.t_begin;
+        if (tt >= 0) {
+            if (first) cp_async_wait_group<0>();
+            else cp_async_wait_group<1>();
         }
+        __syncthreads();                                                            // C0
+        if (tt >= 0 && first) issue_v(t0);   // every thread is done reading the state buffer
         // Rows: thread (i, half hh) takes tokens 8 hh .. 8 hh + 7 of key row i.  The halves
         // exchange through shared memory the first half's decay product and EMA state (for
         // the second) and the second half's decay product (for the first half's end-of-block
@@ -350,6 +364,8 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
         if (tid == 0) {
             tc::fence_after_sync();
             constexpr uint32_t idW = tc::idesc_tf32(128, 2 * L);
+            // A and M need rows 0..L-1 of the product only: M = 64 (rows 0..15 land in lanes 0..15)
+            constexpr uint32_t idAM = tc::idesc_tf32(64, 2 * L);
             // a K-step advances the start addresses (16-byte units, bits 0-13) by two K-chunks
             constexpr uint64_t kStepW = (2 * G::kLboW) >> 4, kStepH = (2 * G::kLboH) >> 4;
             uint64_t bh = tc::smem_desc(tc::smem_addr(bw_hi), G::kLboW, G::kSboW);
@@ -359,12 +375,14 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
 #pragma unroll
             for (int ks = 0; ks < D / 8; ++ks) {
                 const uint32_t acc = ks > 0 ? 1u : 0u;
+                // consecutive products go to different accumulators, so that each waits on a
+                // product issued two places earlier
                 tc::mma_tf32_ts(tmem + G::kDW, tmem + G::kHi + 8 * ks, bh, idW, acc);
+                tc::mma_tf32_ss(tmem + G::kAM, ah, bh, idAM, acc);
                 tc::mma_tf32_ts(tmem + G::kDWc, tmem + G::kHi + 8 * ks, bl, idW, acc);
+                tc::mma_tf32_ss(tmem + G::kAM, ah, bl, idAM, 1u);
                 tc::mma_tf32_ts(tmem + G::kDWc, tmem + G::kLo + 8 * ks, bh, idW, 1u);
-                tc::mma_tf32_ss(tmem + G::kAM, ah, bh, idW, acc);
-                tc::mma_tf32_ss(tmem + G::kAM, ah, bl, idW, 1u);
-                tc::mma_tf32_ss(tmem + G::kAM, al, bh, idW, 1u);
+                tc::mma_tf32_ss(tmem + G::kAM, al, bh, idAM, 1u);
                 bh += kStepW;
                 bl += kStepW;
                 ah += kStepH;
@@ -375,6 +393,11 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
         // the rows are prepared: the next block's k, q, rates and beta can come in
         if (tt >= 0 && !last) issue_kqs(t0 + L);
         wait_mma();
+        // this block's v has landed (the next block's k, q, rates and beta may be in flight)
+        if (tt >= 0) {
+            if (last) cp_async_wait_group<0>();
+            else cp_async_wait_group<1>();
+        }
         if (warp == 0) {
             // A and M to shared memory (lane s < L holds row s of the product)
             float x[L], y[L];
@@ -397,10 +420,18 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
 #pragma unroll
             for (int t = 0; t < L; ++t) {
                 float pp = __fadd_rn(wk[t], ck[t]);
+                // row t of A, four entries per load
 #pragma unroll
-                for (int s = 0; s < t; ++s) pp = fmaf(amA[t * L + s], u[s], pp);
+                for (int s4 = 0; s4 < t; s4 += 4) {
+                    const float4 a4 = reinterpret_cast<const float4*>(amA + t * L)[s4 / 4];
+                    const float av[4] = {a4.x, a4.y, a4.z, a4.w};
+#pragma unroll
+                    for (int e = 0; e < 4; ++e)
+                        if (s4 + e < t) pp = fmaf(av[e], u[s4 + e], pp);
+                }
                 const float bt = p.erase ? sbeta[t] : 1.0f;
-                u[t] = t < n ? (p.erase ? __fsub_rn(__fmul_rn(bt, vv[t]), pp) : vv[t]) : 0.0f;
+                const float vj = sbuf[t * D + jl];
+                u[t] = t < n ? (p.erase ? __fsub_rn(__fmul_rn(bt, vj), pp) : vj) : 0.0f;
             }
             float uh[L], ul[L];
 #pragma unroll
@@ -414,6 +445,7 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
         }
         tc::fence_before_sync();
         __syncthreads();                                                            // C3
+        if (tt >= 0 && !last) issue_v(t0 + L);   // the solve is done with this block's v
 
         // update = u^T (k o Dc_{L-1} / Dc) on the tensor cores (3xTF32, K = 16 tokens)
         if (tid == 0) {
@@ -435,16 +467,22 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
         if (hf == 0) {
             // readouts of column j: o_t = (S_b^T (q o Dc))_t + sum_{s<=t} M_ts u_s, with u from
             // its hi / lo parts in TMEM (written by the value-column thread of the same lane)
-            float wq[L], cq[L], uh[L], ul[L];
+            float wq[L], cq[L], u[L], ul[L];
             tc::tmem_ld2x16(tl + G::kDW + L, tl + G::kDWc + L, wq, cq);
-            tc::tmem_ld2x16(tl + G::kUHi, tl + G::kULo, uh, ul);
+            tc::tmem_ld2x16(tl + G::kUHi, tl + G::kULo, u, ul);
+#pragma unroll
+            for (int t = 0; t < L; ++t) u[t] = __fadd_rn(u[t], ul[t]);
 #pragma unroll
             for (int t = 0; t < L; ++t) {
                 float oa = __fadd_rn(wq[t], cq[t]), ob = 0.0f;
+                // row t of M, four entries per load
 #pragma unroll
-                for (int s = 0; s <= t; s += 2) {
-                    oa = fmaf(amM[t * L + s], __fadd_rn(uh[s], ul[s]), oa);
-                    if (s + 1 <= t) ob = fmaf(amM[t * L + s + 1], __fadd_rn(uh[s + 1], ul[s + 1]), ob);
+                for (int s4 = 0; s4 <= t; s4 += 4) {
+                    const float4 m4 = reinterpret_cast<const float4*>(amM + t * L)[s4 / 4];
+                    if (s4 <= t) oa = fmaf(m4.x, u[s4], oa);
+                    if (s4 + 1 <= t) ob = fmaf(m4.y, u[s4 + 1], ob);
+                    if (s4 + 2 <= t) oa = fmaf(m4.z, u[s4 + 2], oa);
+                    if (s4 + 3 <= t) ob = fmaf(m4.w, u[s4 + 3], ob);
                 }
                 if (t < n) p.o[((tokb + t0 + t) * p.H + h) * D + jl] = oa + ob;
             }
