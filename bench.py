@@ -278,6 +278,9 @@ def main():
     w = synth.WORKLOADS[args.workload]
     if args.T:
         w = synth.scaled(w, T=args.T)
+    if args.form == "auto":
+        args.form = ("chunk" if w.C > 1 and w.unit == "row" and w.dk == 128 and w.dv == 128
+                     and not w.general else "token")
     if args.impl == "reference":
         return run_reference(args, w)
 
@@ -295,9 +298,6 @@ def main():
     torch.cuda.set_device(dev)
     q.load(build_if_missing=True)
 
-    if args.form == "auto":
-        args.form = ("chunk" if w.C > 1 and w.unit == "row" and w.dk == 128 and w.dv == 128
-                     and not w.general else "token")
     cfg = q.Config.from_workload(w, fit_every=args.fit_every, alloc_mode=args.alloc_mode,
                                  interval_form=q.FORM_CHUNK if args.form == "chunk" else q.FORM_TOKEN)
     x = synth.device_inputs(w, device=dev, seed_offset=rank_seed_offset(rank))
