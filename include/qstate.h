@@ -181,8 +181,9 @@ double qstate_bits_per_element(const qstate_cfg* cfg);
  * (scales 0, factor index 15).  `b` receives the same widths and offsets. */
 int qstate_init(const qstate_cfg* cfg, qstate_buf* a, qstate_buf* b, void* stream);
 
-/* Sec. 3, Eq. (3) and Eq. (4) + "round, clip to [b_min, b_max], and adjust widths to meet the
- * layer budget": per batch element, weights c_i = Gamma_hat_i Rtilde_i^2 from `stats`
+/* Sec. 3, Eq. (3) and Eq. (4), followed by the paper's integer step (the real widths are
+ * rounded, limited to [b_min, b_max] and corrected until they sum to the layer budget): per
+ * batch element, weights c_i = Gamma_hat_i Rtilde_i^2 from `stats`
  * (Gamma_hat = (1 - ema_s)/(expm1(ema_r) + ema_s), Rtilde_i^2 = R_i^2 / mean over the group of
  * R^2, 1 for the head unit) and integer widths summing exactly to units*bbar: the widths that
  * minimise sum_i c_i 4^{-w_i} under the limits, ties going to lower unit indices.  Writes
