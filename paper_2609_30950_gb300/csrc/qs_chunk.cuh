@@ -237,33 +237,39 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
         float kk[LH], dd[LH], pr[LH], sf[LH];
         {
             float xs[LH], xr[LH], qv[LH], bv[LH];
+            // branch-free over the half's tokens (tokens past n read staged bytes of earlier
+            // blocks, in bounds, and are masked), so the eight exp / expm1 chains interleave
+            bool bad = false;
 #pragma unroll
             for (int j = 0; j < LH; ++j) {
                 const int tau = tb + j;
-                kk[j] = qv[j] = bv[j] = xs[j] = xr[j] = 0.0f;
-                dd[j] = 1.0f;
-                if (tau < n) {
-                    kk[j] = sk[tau * D + i];
-                    qv[j] = sq[tau * D + i];
-                    if (p.erase) bv[j] = sbeta[tau];
-                    float rate;
-                    if (!p.decay_row) {
-                        rate = ss[tau];
-                    } else if (p.s_code) {
-                        const int code = min(static_cast<int>(sc[tau * D + i]), p.L - 1);
-                        rate = p.L <= 4 ? S.lut[i * p.L + code]
-                                        : __ldg(p.s_lut + (static_cast<size_t>(h) * D + i) * p.L + code);
-                    } else {
-                        rate = ss[tau * D + i];
-                    }
-                    if (!(rate > 0.0f) || !(rate < INFINITY)) raise_status(p.status, QS_DEV_RATE);
-                    dd[j] = expf(-rate);
-                    if (stats) {
-                        xs[j] = -expm1f(-2.0f * rate);
-                        xr[j] = p.erase ? __fmul_rn(__fmul_rn(bv[j], __fsub_rn(2.0f, bv[j])), __fmul_rn(kk[j], kk[j])) : 0.0f;
-                    }
+                const bool live = tau < n;
+                float rate;
+                if (!p.decay_row) {
+                    rate = ss[tau];
+                } else if (p.s_code) {
+                    const int code = min(static_cast<int>(sc[tau * D + i]), p.L - 1);
+                    rate = p.L <= 4 ? S.lut[i * p.L + code]
+                                    : __ldg(p.s_lut + (static_cast<size_t>(h) * D + i) * p.L + code);
+                } else {
+                    rate = ss[tau * D + i];
+                }
+                bad |= live && (!(rate > 0.0f) || !(rate < INFINITY));
+                rate = live ? rate : 1.0f;
+                const float kq = sk[tau * D + i], qq = sq[tau * D + i];
+                const float bq = p.erase ? sbeta[tau] : 0.0f;
+                kk[j] = live ? kq : 0.0f;
+                qv[j] = live ? qq : 0.0f;
+                bv[j] = live ? bq : 0.0f;
+                const float d = expf(-rate);
+                dd[j] = live ? d : 1.0f;
+                xs[j] = xr[j] = 0.0f;
+                if (stats) {
+                    xs[j] = -expm1f(-2.0f * rate);
+                    xr[j] = p.erase ? __fmul_rn(__fmul_rn(bv[j], __fsub_rn(2.0f, bv[j])), __fmul_rn(kk[j], kk[j])) : 0.0f;
                 }
             }
+            if (bad) raise_status(p.status, QS_DEV_RATE);
             // decay products within the half: pr[j] = d_tb ... d_{tb+j}, sf[j] = d_{tb+j+1} ... d_{tb+LH-1}
             float acc = 1.0f;
 #pragma unroll
