@@ -32,6 +32,11 @@ CASES = {
     # no erasure (a = 0, w = 1), per-head rates, 128 x 128
     "mamba_128_c32": (lambda: synth.scaled(synth.WORKLOADS["mamba2_decode"], B=2, H=8, T=70, C=32,
                                            dv=128, group_heads=4), False),
+    # log-quantised rates with 8 levels (level table read from global memory)
+    "decode_coded_g3_c48": (lambda: small("kda_decode", B=2, H=3, T=70, C=48, gate_bits=3), True),
+    # per-head log-quantised rates, row unit
+    "gdn_row_coded_c32": (lambda: synth.scaled(synth.WORKLOADS["gdn_decode"], B=2, H=4, T=45, C=32,
+                                               unit="row", bmin=1, bmax=8, gate_bits=2), True),
     # slow channels that keep their rate over the whole sequence
     "persistent_c64": (lambda: synth.scaled(synth.EXTENSION_WORKLOADS["kda_persistent"], B=2, H=3,
                                             T=130, C=64), True),
