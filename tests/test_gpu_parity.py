@@ -354,15 +354,15 @@ def test_persistent_decay_lockstep(qs, orc):
     _lockstep(qs, orc, w, log_decay=True)
 
 
-@pytest.mark.parametrize("name,log_decay", [("kda_decode", True), ("mamba2_decode", False),
-                                            ("kda_prefill", False)])
-def test_current_allocation_lockstep(qs, orc, name, log_decay):
+@pytest.mark.parametrize("name,log_decay,form", [("kda_decode", True, 0), ("mamba2_decode", False, 0),
+                                                 ("kda_prefill", False, 0), ("kda_prefill", False, 1)])
+def test_current_allocation_lockstep(qs, orc, name, log_decay, form):
     """alloc_mode current: each write-back allocates from its own statistics (a statistics
     pass, the allocation, then the packing pass).  The oracle runs free; before every
     write-back its state is copied into the GPU; widths, codes, readouts and statistics of the
-    GPU's write-back are compared with the oracle's."""
+    GPU's write-back are compared with the oracle's.  form 1: both passes in chunked form."""
     w = SMALL[name]
-    cfgq = qs.Config.from_workload(w, alloc_mode=1)
+    cfgq = qs.Config.from_workload(w, alloc_mode=1, interval_form=form)
     cfgo = orc.Cfg.from_workload(w, alloc_mode=1)
     inp = synth.host_inputs(w)
     s_code = s_lut = None
