@@ -470,9 +470,10 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
             }
             tc::mma_commit(bar);
         }
-        if (hf == 0) {
+        {
             // readouts of column j: o_t = (S_b^T (q o Dc))_t + sum_{s<=t} M_ts u_s, with u from
-            // its hi / lo parts in TMEM (written by the value-column thread of the same lane)
+            // its hi / lo parts in TMEM; warps 0-3 take tokens 0..7, warps 4-7 tokens 8..15 of
+            // the same columns (the same TMEM lanes)
             float wq[L], cq[L], u[L], ul[L];
             tc::tmem_ld2x16(tl + G::kDW + L, tl + G::kDWc + L, wq, cq);
             tc::tmem_ld2x16(tl + G::kUHi, tl + G::kULo, u, ul);
@@ -480,6 +481,7 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
             for (int t = 0; t < L; ++t) u[t] = __fadd_rn(u[t], ul[t]);
 #pragma unroll
             for (int t = 0; t < L; ++t) {
+                if ((t >= L / 2) != (hf == 1)) continue;
                 float oa = __fadd_rn(wq[t], cq[t]), ob = 0.0f;
                 // row t of M, four entries per load
 #pragma unroll
@@ -499,8 +501,7 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
 #pragma unroll 1
         for (int c0 = 64 * hf; c0 < 64 * hf + 64; c0 += 16) {
             float hi[16], lo[16], up[16];
-            tc::tmem_ld2x16(tl + G::kHi + c0, tl + G::kLo + c0, hi, lo);
-            tc::tmem_ld16(tl + G::kUpd + c0, up);
+            tc::tmem_ld3x16(tl + G::kHi + c0, tl + G::kLo + c0, tl + G::kUpd + c0, hi, lo, up);
 #pragma unroll
             for (int c = 0; c < 16; ++c) {
                 const float x = fmaf(__fadd_rn(hi[c], lo[c]), dall[c0 + c], up[c]);
