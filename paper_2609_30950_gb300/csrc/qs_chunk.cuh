@@ -26,10 +26,10 @@
 // over 16 tokens; a block beyond that raises QS_DEV_CHUNK (the token-by-token kernel has no such
 // limit).
 //
-// Roles per block (256 threads): warps 0-3 own key rows (thread = row i): rates, decays, EMA
-// statistics and the operand tiles, and later value columns for the readouts; warps 4-7 stage
-// the next block's inputs and own value columns (TMEM lane j) for the solve.  All threads
-// combine and split the state.
+// Roles per block (256 threads): thread (row i, half) prepares key row i for 8 of the block's
+// 16 tokens (rates, decays, EMA statistics, operand tiles); warps 4-7 also stage the next
+// block's inputs and own value columns (TMEM lane j) for the solve; the readouts are split
+// over both halves by token; all threads combine and split the state.
 // Included by qs_wb_row.cuh, whose state-buffer swizzle sb_off it uses.
 #pragma once
 
