@@ -75,15 +75,17 @@ struct ChunkGeo {
     static constexpr uint32_t oKhHi = 0, oKhLo = kKh, oBwHi = 2 * kKh, oBwLo = 2 * kKh + kBw;
     static constexpr uint32_t oBuHi = 2 * kKh + 2 * kBw, oBuLo = oBuHi + kBu;
     static constexpr uint32_t oAM = oBuLo + kBu;                  // A and M, L x L each
-    static constexpr uint32_t oDall = oAM + 2 * L * L * 4;
-    static constexpr uint32_t oXch = oDall + D * 4;              // row preparation: the halves' exchange
-    static constexpr uint32_t oBar = oXch + 2 * D * 16;          // mbarrier (8 bytes) + TMEM address
-    // one block's token inputs, staged by cp.async one block ahead: k, q, rates (FP32 per row,
-    // per head, or uint8 codes) and beta (two buffers by block parity: the solve of block c
-    // still reads its beta when block c + 1's arrives)
-    static constexpr uint32_t oStg = oBar + 16;
+    static constexpr uint32_t oDall = oAM + 2 * L * L * 4;        // two buffers, by block parity
+    static constexpr uint32_t oXch = oDall + 2 * D * 4;          // row preparation: the halves' exchange
+    // mbarriers of the products with S_b and A / M (two arrivals) and of the update (one),
+    // then the TMEM address
+    static constexpr uint32_t oBar = oXch + 2 * D * 16;
+    // one block's token inputs, staged by cp.async: k, q, rates (FP32 per row, per head, or
+    // uint8 codes) and beta (three buffers by block index mod 3: block c's solve still reads
+    // its beta while block c + 2's arrives)
+    static constexpr uint32_t oStg = oBar + 32;
     static constexpr uint32_t sK = 0, sQ = L * D * 4, sS = 2 * L * D * 4, sB = 3 * L * D * 4;
-    static constexpr uint32_t kBytes = oStg + sB + 2 * L * 4;
+    static constexpr uint32_t kBytes = oStg + sB + 3 * L * 4;
     static constexpr int kWaitPolls = 1 << 24;
 };
 static_assert(ChunkGeo::oBwHi % 16 == 0 && ChunkGeo::oBuHi % 16 == 0 && ChunkGeo::oBar % 16 == 0 &&
@@ -99,13 +101,14 @@ __device__ __forceinline__ uint32_t chunk_setup(uint8_t* cb) {
     using G = ChunkGeo;
     const int tid = threadIdx.x;
     uint64_t* bar = reinterpret_cast<uint64_t*>(cb + G::oBar);
-    uint32_t* ta = reinterpret_cast<uint32_t*>(cb + G::oBar + 8);
+    uint32_t* ta = reinterpret_cast<uint32_t*>(cb + G::oBar + 16);
     if (tid < 32) {
         tc::tmem_alloc(ta, G::kCols);
         tc::tmem_relinquish();
     }
     if (tid == 32) {
-        tc::mbar_init(bar, 1);
+        tc::mbar_init(bar, 2);       // products with S_b (thread 0) and for A / M (thread 32)
+        tc::mbar_init(bar + 1, 1);   // the update
         tc::mbar_fence_init();
     }
     tc::fence_before_sync();
@@ -125,7 +128,7 @@ __device__ __forceinline__ void chunk_teardown(uint32_t tmem) {
 
 // The interval [p.t_begin, p.t_end) of head (b, h): the state arrives in sbuf (row-major,
 // swizzled) and leaves there; readouts go to p.o, the EMA statistics of the rows to S.ms / S.mr.
-// `phase` tracks the mbarrier's parity (uniform over the CTA).
+// `phase` tracks the mbarriers' parities (uniform over the CTA).
 template <class Stage>
 __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, float* sbuf, uint8_t* cb,
                                                uint32_t tmem, uint32_t& phase, int b, int h, bool stats) {
@@ -152,16 +155,17 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
     const float* ss = reinterpret_cast<const float*>(stg + G::sS);
     const uint8_t* sc = stg + G::sS;
     const size_t tokb = static_cast<size_t>(b) * p.T;
-    auto wait_mma = [&]() {
-        if (!tc::mbar_wait(bar, phase, G::kWaitPolls)) raise_status(p.status, QS_DEV_TIMEOUT);
-        phase ^= 1u;
+    // `phase` carries both mbarriers' parities: bit 0 the first's, bit 1 the second's
+    auto wait_mma = [&](int which) {
+        if (!tc::mbar_wait(bar + which, (phase >> which) & 1u, G::kWaitPolls)) raise_status(p.status, QS_DEV_TIMEOUT);
+        phase ^= 1u << which;
         tc::fence_after_sync();
     };
     // staging of the block at token tb by the value-column threads: k, q, the rates and beta
     auto issue_kqs = [&](int tb) {
         const int nb = min(L, p.t_end - tb);
         if (p.erase && tt < nb)
-            cp_async4(stg + G::sB + (((tb - p.t_begin) / L) & 1) * L * 4 + tt * 4, p.beta + (tokb + tb + tt) * p.H + h);
+            cp_async4(stg + G::sB + (((tb - p.t_begin) / L) % 3) * L * 4 + tt * 4, p.beta + (tokb + tb + tt) * p.H + h);
         for (int c = tt; c < nb * (D / 4); c += 128) {
             const int tau = c / (D / 4), part = c % (D / 4);
             const size_t tok = (tokb + tb + tau) * p.H + h;
@@ -213,161 +217,180 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
     tc::wait_st();
     tc::fence_before_sync();
 
+    // Rows: thread (i, half hh) takes tokens 8 hh .. 8 hh + 7 of key row i.  Phase A (staged
+    // loads, decays, EMA terms, the first half's EMA recursion) of block c + 1 runs while the
+    // tensor cores work on block c; phase B (the second half's EMA recursion, cumulative decays,
+    // operand tiles) at the start of block c + 1.  The halves exchange through shared memory the
+    // first half's decay product and EMA state and the second half's decay product.
+    constexpr int LH = L / 2;
+    const int i = tid & (D - 1), hh = tid >> 7, tb = LH * hh;
+    float4* xch = reinterpret_cast<float4*>(cb + G::oXch);
+    struct RowA {
+        float kk[LH], dd[LH], qv[LH], bv[LH], xs[LH], xr[LH];
+    };
+    auto phase_a = [&](int t0b, RowA& r) {
+        const int nb = min(L, p.t_end - t0b);
+        const float* sbeta = reinterpret_cast<const float*>(stg + G::sB) + (((t0b - p.t_begin) / L) % 3) * L;
+        // branch-free over the half's tokens (tokens past nb read staged bytes of earlier
+        // blocks, in bounds, and are masked), so the eight exp / expm1 chains interleave
+        bool bad = false;
+#pragma unroll
+        for (int j = 0; j < LH; ++j) {
+            const int tau = tb + j;
+            const bool live = tau < nb;
+            float rate;
+            if (!p.decay_row) {
+                rate = ss[tau];
+            } else if (p.s_code) {
+                const int code = min(static_cast<int>(sc[tau * D + i]), p.L - 1);
+                rate = p.L <= 4 ? S.lut[i * p.L + code]
+                                : __ldg(p.s_lut + (static_cast<size_t>(h) * D + i) * p.L + code);
+            } else {
+                rate = ss[tau * D + i];
+            }
+            bad |= live && (!(rate > 0.0f) || !(rate < INFINITY));
+            rate = live ? rate : 1.0f;
+            const float kq = sk[tau * D + i], qq = sq[tau * D + i];
+            const float bq = p.erase ? sbeta[tau] : 0.0f;
+            r.kk[j] = live ? kq : 0.0f;
+            r.qv[j] = live ? qq : 0.0f;
+            r.bv[j] = live ? bq : 0.0f;
+            const float d = expf(-rate);
+            r.dd[j] = live ? d : 1.0f;
+            r.xs[j] = r.xr[j] = 0.0f;
+            if (stats) {
+                r.xs[j] = -expm1f(-2.0f * rate);
+                r.xr[j] = p.erase ? __fmul_rn(__fmul_rn(r.bv[j], __fsub_rn(2.0f, r.bv[j])), __fmul_rn(r.kk[j], r.kk[j])) : 0.0f;
+            }
+        }
+        if (bad) raise_status(p.status, QS_DEV_RATE);
+        float prod = 1.0f;
+#pragma unroll
+        for (int j = 0; j < LH; ++j) prod = __fmul_rn(prod, r.dd[j]);
+        if (hh == 0) {
+            // the EMA recursion over the first half (from the state after the previous block)
+            float ms = stats ? S.ms[i] : 0.0f, mr = stats ? S.mr[i] : 0.0f;
+            if (stats) {
+#pragma unroll
+                for (int j = 0; j < LH; ++j) {
+                    if (j >= nb) break;
+                    if (t0b + j == 0) {
+                        ms = r.xs[j];
+                        mr = r.xr[j];
+                    } else {
+                        ms = __fadd_rn(ms, __fmul_rn(p.alpha, __fsub_rn(r.xs[j], ms)));
+                        mr = __fadd_rn(mr, __fmul_rn(p.alpha, __fsub_rn(r.xr[j], mr)));
+                    }
+                }
+            }
+            xch[i] = make_float4(prod, ms, mr, 0.0f);
+        } else {
+            xch[D + i].x = prod;
+        }
+    };
+    auto phase_b = [&](int t0b, const RowA& r) {
+        const int nb = min(L, p.t_end - t0b);
+        float* dl = dall + (((t0b - p.t_begin) / L) & 1) * D;
+        float pr[LH], sf[LH];
+        float acc = 1.0f;
+#pragma unroll
+        for (int j = 0; j < LH; ++j) pr[j] = acc = __fmul_rn(acc, r.dd[j]);
+        acc = 1.0f;
+#pragma unroll
+        for (int j = LH - 1; j >= 0; --j) {
+            sf[j] = acc;
+            acc = __fmul_rn(acc, r.dd[j]);
+        }
+        const float4 x0 = xch[i];
+        const float dc0 = hh == 0 ? 1.0f : x0.x;            // decay before the half
+        const float sf1 = hh == 0 ? xch[D + i].x : 1.0f;   // decay after the half, in the block
+        if (hh == 1) {
+            // the EMA state after the whole block and the block's decay (with no second-half
+            // tokens, the first half's)
+            float ms = x0.y, mr = x0.z;
+            if (stats) {
+#pragma unroll
+                for (int j = 0; j < LH; ++j) {
+                    if (tb + j >= nb) break;
+                    ms = __fadd_rn(ms, __fmul_rn(p.alpha, __fsub_rn(r.xs[j], ms)));
+                    mr = __fadd_rn(mr, __fmul_rn(p.alpha, __fsub_rn(r.xr[j], mr)));
+                }
+                S.ms[i] = ms;
+                S.mr[i] = mr;
+            }
+            const float Dall = __fmul_rn(dc0, pr[LH - 1]);
+            if (!(Dall >= 1e-37f)) raise_status(p.status, QS_DEV_CHUNK);
+            dl[i] = Dall;
+        }
+        const int oh = (i >> 2) * G::kLboH + (i & 3) * 4, ow = (i >> 2) * G::kLboW + (i & 3) * 4;
+#pragma unroll
+        for (int j = 0; j < LH; ++j) {
+            const int tau = tb + j;
+            const float Dc = __fmul_rn(dc0, pr[j]);
+            const float a = p.erase ? __fmul_rn(r.bv[j], r.kk[j]) : 0.0f;
+            const float kt = __fmul_rn(a, Dc), qt = __fmul_rn(r.qv[j], Dc);
+            float rDc;   // k / Dc only enters A and M
+            asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(rDc) : "f"(Dc));
+            const float kh = tau < nb ? __fmul_rn(r.kk[j], rDc) : 0.0f;
+            // tiles: k / Dc row tau; [a o Dc ; q o Dc] rows tau and L + tau (row r of a
+            // K-chunk at byte 16 r)
+            const float khh = tc::tf32_hi(kh), kth = tc::tf32_hi(kt), qth = tc::tf32_hi(qt);
+            *reinterpret_cast<float*>(kh_hi + oh + 16 * tau) = khh;
+            *reinterpret_cast<float*>(kh_lo + oh + 16 * tau) = __fsub_rn(kh, khh);
+            *reinterpret_cast<float*>(bw_hi + ow + 16 * tau) = kth;
+            *reinterpret_cast<float*>(bw_lo + ow + 16 * tau) = __fsub_rn(kt, kth);
+            *reinterpret_cast<float*>(bw_hi + ow + 16 * (L + tau)) = qth;
+            *reinterpret_cast<float*>(bw_lo + ow + 16 * (L + tau)) = __fsub_rn(qt, qth);
+        }
+        // (k o Dc_{L-1} / Dc)^T: row i, tokens of the half, 4 per 16-byte chunk
+#pragma unroll
+        for (int c4 = 0; c4 < LH / 4; ++c4) {
+            float kb[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) kb[e] = __fmul_rn(r.kk[4 * c4 + e], __fmul_rn(sf[4 * c4 + e], sf1));
+            float4 hi, lo;
+            hi.x = tc::tf32_hi(kb[0]);
+            hi.y = tc::tf32_hi(kb[1]);
+            hi.z = tc::tf32_hi(kb[2]);
+            hi.w = tc::tf32_hi(kb[3]);
+            lo.x = __fsub_rn(kb[0], hi.x);
+            lo.y = __fsub_rn(kb[1], hi.y);
+            lo.z = __fsub_rn(kb[2], hi.z);
+            lo.w = __fsub_rn(kb[3], hi.w);
+            const int o = ((tb >> 2) + c4) * G::kLboU + (i >> 3) * G::kSboU + (i & 7) * 16;
+            *reinterpret_cast<float4*>(bu_hi + o) = hi;
+            *reinterpret_cast<float4*>(bu_lo + o) = lo;
+        }
+    };
+
+    RowA ra;   // phase A of the block about to start
+    if (p.t_begin < p.t_end) {
+        if (tt >= 0) cp_async_wait_all();
+        __syncthreads();                      // the first block's inputs; the state buffer is read
+        if (tt >= 0) issue_v(p.t_begin);
+        phase_a(p.t_begin, ra);
+        __syncthreads();                      // the first block's exchange; its staging is read
+        if (tt >= 0 && p.t_begin + L < p.t_end) issue_kqs(p.t_begin + L);
+    }
+
 #pragma unroll 1
     for (int t0 = p.t_begin; t0 < p.t_end; t0 += L) {
         const int n = min(L, p.t_end - t0);
         const bool last = t0 + L >= p.t_end;
-        const float* sbeta = reinterpret_cast<const float*>(stg + G::sB) + (((t0 - p.t_begin) / L) & 1) * L;
-        // this block's k, q, rates and beta have landed (the first block's v is not yet asked for;
-        // a later block's may still be in flight)
-        const bool first = t0 == p.t_begin;
-        if (tt >= 0) {
-            if (first) cp_async_wait_group<0>();
-            else cp_async_wait_group<1>();
-        }
-        __syncthreads();                                                            // C0
-        if (tt >= 0 && first) issue_v(t0);   // every thread is done reading the state buffer
-        // Rows: thread (i, half hh) takes tokens 8 hh .. 8 hh + 7 of key row i.  The halves
-        // exchange through shared memory the first half's decay product and EMA state (for
-        // the second) and the second half's decay product (for the first half's end-of-block
-        // factors); the EMA recursion runs token by token in order.
-        constexpr int LH = L / 2;
-        const int i = tid & (D - 1), hh = tid >> 7, tb = LH * hh;
-        float4* xch = reinterpret_cast<float4*>(cb + G::oXch);
-        float kk[LH], dd[LH], pr[LH], sf[LH];
-        {
-            float xs[LH], xr[LH], qv[LH], bv[LH];
-            // branch-free over the half's tokens (tokens past n read staged bytes of earlier
-            // blocks, in bounds, and are masked), so the eight exp / expm1 chains interleave
-            bool bad = false;
-#pragma unroll
-            for (int j = 0; j < LH; ++j) {
-                const int tau = tb + j;
-                const bool live = tau < n;
-                float rate;
-                if (!p.decay_row) {
-                    rate = ss[tau];
-                } else if (p.s_code) {
-                    const int code = min(static_cast<int>(sc[tau * D + i]), p.L - 1);
-                    rate = p.L <= 4 ? S.lut[i * p.L + code]
-                                    : __ldg(p.s_lut + (static_cast<size_t>(h) * D + i) * p.L + code);
-                } else {
-                    rate = ss[tau * D + i];
-                }
-                bad |= live && (!(rate > 0.0f) || !(rate < INFINITY));
-                rate = live ? rate : 1.0f;
-                const float kq = sk[tau * D + i], qq = sq[tau * D + i];
-                const float bq = p.erase ? sbeta[tau] : 0.0f;
-                kk[j] = live ? kq : 0.0f;
-                qv[j] = live ? qq : 0.0f;
-                bv[j] = live ? bq : 0.0f;
-                const float d = expf(-rate);
-                dd[j] = live ? d : 1.0f;
-                xs[j] = xr[j] = 0.0f;
-                if (stats) {
-                    xs[j] = -expm1f(-2.0f * rate);
-                    xr[j] = p.erase ? __fmul_rn(__fmul_rn(bv[j], __fsub_rn(2.0f, bv[j])), __fmul_rn(kk[j], kk[j])) : 0.0f;
-                }
-            }
-            if (bad) raise_status(p.status, QS_DEV_RATE);
-            // decay products within the half: pr[j] = d_tb ... d_{tb+j}, sf[j] = d_{tb+j+1} ... d_{tb+LH-1}
-            float acc = 1.0f;
-#pragma unroll
-            for (int j = 0; j < LH; ++j) pr[j] = acc = __fmul_rn(acc, dd[j]);
-            acc = 1.0f;
-#pragma unroll
-            for (int j = LH - 1; j >= 0; --j) {
-                sf[j] = acc;
-                acc = __fmul_rn(acc, dd[j]);
-            }
-            if (hh == 0) {
-                float ms = stats ? S.ms[i] : 0.0f, mr = stats ? S.mr[i] : 0.0f;
-                if (stats) {
-#pragma unroll
-                    for (int j = 0; j < LH; ++j) {
-                        if (j >= n) break;
-                        if (t0 + j == 0) {
-                            ms = xs[j];
-                            mr = xr[j];
-                        } else {
-                            ms = __fadd_rn(ms, __fmul_rn(p.alpha, __fsub_rn(xs[j], ms)));
-                            mr = __fadd_rn(mr, __fmul_rn(p.alpha, __fsub_rn(xr[j], mr)));
-                        }
-                    }
-                }
-                xch[i] = make_float4(pr[LH - 1], ms, mr, 0.0f);
-            } else {
-                xch[D + i].x = pr[LH - 1];
-            }
-            __syncthreads();                                                        // Cx
-            const float4 x0 = xch[i];
-            const float dc0 = hh == 0 ? 1.0f : x0.x;            // decay before the half
-            const float sf1 = hh == 0 ? xch[D + i].x : 1.0f;   // decay after the half, in the block
-            if (hh == 1) {
-                // the EMA state after the whole block and the block's decay (with no second-half
-                // tokens, the first half's)
-                float ms = x0.y, mr = x0.z;
-                if (stats) {
-#pragma unroll
-                    for (int j = 0; j < LH; ++j) {
-                        if (tb + j >= n) break;
-                        ms = __fadd_rn(ms, __fmul_rn(p.alpha, __fsub_rn(xs[j], ms)));
-                        mr = __fadd_rn(mr, __fmul_rn(p.alpha, __fsub_rn(xr[j], mr)));
-                    }
-                    S.ms[i] = ms;
-                    S.mr[i] = mr;
-                }
-                const float Dall = __fmul_rn(dc0, pr[LH - 1]);
-                if (!(Dall >= 1e-37f)) raise_status(p.status, QS_DEV_CHUNK);
-                dall[i] = Dall;
-            }
-            const int oh = (i >> 2) * G::kLboH + (i & 3) * 4, ow = (i >> 2) * G::kLboW + (i & 3) * 4;
-#pragma unroll
-            for (int j = 0; j < LH; ++j) {
-                const int tau = tb + j;
-                const float Dc = __fmul_rn(dc0, pr[j]);
-                const float a = p.erase ? __fmul_rn(bv[j], kk[j]) : 0.0f;
-                const float kt = __fmul_rn(a, Dc), qt = __fmul_rn(qv[j], Dc);
-                float rDc;   // k / Dc only enters A and M
-                asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(rDc) : "f"(Dc));
-                const float kh = tau < n ? __fmul_rn(kk[j], rDc) : 0.0f;
-                // tiles: k / Dc row tau; [a o Dc ; q o Dc] rows tau and L + tau (row r of a
-                // K-chunk at byte 16 r)
-                const float khh = tc::tf32_hi(kh), kth = tc::tf32_hi(kt), qth = tc::tf32_hi(qt);
-                *reinterpret_cast<float*>(kh_hi + oh + 16 * tau) = khh;
-                *reinterpret_cast<float*>(kh_lo + oh + 16 * tau) = __fsub_rn(kh, khh);
-                *reinterpret_cast<float*>(bw_hi + ow + 16 * tau) = kth;
-                *reinterpret_cast<float*>(bw_lo + ow + 16 * tau) = __fsub_rn(kt, kth);
-                *reinterpret_cast<float*>(bw_hi + ow + 16 * (L + tau)) = qth;
-                *reinterpret_cast<float*>(bw_lo + ow + 16 * (L + tau)) = __fsub_rn(qt, qth);
-            }
-            // (k o Dc_{L-1} / Dc)^T: row i, tokens of the half, 4 per 16-byte chunk
-#pragma unroll
-            for (int c4 = 0; c4 < LH / 4; ++c4) {
-                float kb[4];
-#pragma unroll
-                for (int e = 0; e < 4; ++e) kb[e] = __fmul_rn(kk[4 * c4 + e], __fmul_rn(sf[4 * c4 + e], sf1));
-                float4 hi, lo;
-                hi.x = tc::tf32_hi(kb[0]);
-                hi.y = tc::tf32_hi(kb[1]);
-                hi.z = tc::tf32_hi(kb[2]);
-                hi.w = tc::tf32_hi(kb[3]);
-                lo.x = __fsub_rn(kb[0], hi.x);
-                lo.y = __fsub_rn(kb[1], hi.y);
-                lo.z = __fsub_rn(kb[2], hi.z);
-                lo.w = __fsub_rn(kb[3], hi.w);
-                const int o = ((tb >> 2) + c4) * G::kLboU + (i >> 3) * G::kSboU + (i & 7) * 16;
-                *reinterpret_cast<float4*>(bu_hi + o) = hi;
-                *reinterpret_cast<float4*>(bu_lo + o) = lo;
-            }
-        }
+        const float* sbeta = reinterpret_cast<const float*>(stg + G::sB) + (((t0 - p.t_begin) / L) % 3) * L;
+        const float* dall_c = dall + (((t0 - p.t_begin) / L) & 1) * D;
+        phase_b(t0, ra);
+        // the next block's k, q, rates and beta and this block's v have landed
+        if (tt >= 0) cp_async_wait_all();
         tc::fence_async_smem();
         __syncthreads();                                                            // C1
 
-        // On the tensor cores (3xTF32, K = 128 key rows): S_b^T [a o Dc ; q o Dc]^T, its hi*hi
-        // product and the two corrections in separate accumulators, and (k / Dc) [a o Dc ;
-        // q o Dc]^T, whose row s, column t is A_ts (column < L) or M_ts (column >= L)
-        if (tid == 0) {
+        // On the tensor cores (3xTF32, K = 128 key rows), issued by two threads of different
+        // warps (an issuing thread stalls while the product queue is full): thread 0 issues
+        // S_b^T [a o Dc ; q o Dc]^T, its hi*hi product and the two corrections in separate
+        // accumulators; thread 32 issues (k / Dc) [a o Dc ; q o Dc]^T, whose row s, column t is
+        // A_ts (column < L) or M_ts (column >= L)
+        if (tid == 0 || tid == 32) {
             tc::fence_after_sync();
             constexpr uint32_t idW = tc::idesc_tf32(128, 2 * L);
             // A and M need rows 0..L-1 of the product only: M = 64 (rows 0..15 land in lanes 0..15)
@@ -376,34 +399,36 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
             constexpr uint64_t kStepW = (2 * G::kLboW) >> 4, kStepH = (2 * G::kLboH) >> 4;
             uint64_t bh = tc::smem_desc(tc::smem_addr(bw_hi), G::kLboW, G::kSboW);
             uint64_t bl = tc::smem_desc(tc::smem_addr(bw_lo), G::kLboW, G::kSboW);
-            uint64_t ah = tc::smem_desc(tc::smem_addr(kh_hi), G::kLboH, G::kSboH);
-            uint64_t al = tc::smem_desc(tc::smem_addr(kh_lo), G::kLboH, G::kSboH);
+            if (tid == 0) {
 #pragma unroll
-            for (int ks = 0; ks < D / 8; ++ks) {
-                const uint32_t acc = ks > 0 ? 1u : 0u;
-                // consecutive products go to different accumulators, so that each waits on a
-                // product issued two places earlier
-                tc::mma_tf32_ts(tmem + G::kDW, tmem + G::kHi + 8 * ks, bh, idW, acc);
-                tc::mma_tf32_ss(tmem + G::kAM, ah, bh, idAM, acc);
-                tc::mma_tf32_ts(tmem + G::kDWc, tmem + G::kHi + 8 * ks, bl, idW, acc);
-                tc::mma_tf32_ss(tmem + G::kAM, ah, bl, idAM, 1u);
-                tc::mma_tf32_ts(tmem + G::kDWc, tmem + G::kLo + 8 * ks, bh, idW, 1u);
-                tc::mma_tf32_ss(tmem + G::kAM, al, bh, idAM, 1u);
-                bh += kStepW;
-                bl += kStepW;
-                ah += kStepH;
-                al += kStepH;
+                for (int ks = 0; ks < D / 8; ++ks) {
+                    const uint32_t acc = ks > 0 ? 1u : 0u;
+                    tc::mma_tf32_ts(tmem + G::kDW, tmem + G::kHi + 8 * ks, bh, idW, acc);
+                    tc::mma_tf32_ts(tmem + G::kDWc, tmem + G::kHi + 8 * ks, bl, idW, acc);
+                    tc::mma_tf32_ts(tmem + G::kDWc, tmem + G::kLo + 8 * ks, bh, idW, 1u);
+                    bh += kStepW;
+                    bl += kStepW;
+                }
+            } else {
+                uint64_t ah = tc::smem_desc(tc::smem_addr(kh_hi), G::kLboH, G::kSboH);
+                uint64_t al = tc::smem_desc(tc::smem_addr(kh_lo), G::kLboH, G::kSboH);
+#pragma unroll
+                for (int ks = 0; ks < D / 8; ++ks) {
+                    const uint32_t acc = ks > 0 ? 1u : 0u;
+                    tc::mma_tf32_ss(tmem + G::kAM, ah, bh, idAM, acc);
+                    tc::mma_tf32_ss(tmem + G::kAM, ah, bl, idAM, 1u);
+                    tc::mma_tf32_ss(tmem + G::kAM, al, bh, idAM, 1u);
+                    bh += kStepW;
+                    bl += kStepW;
+                    ah += kStepH;
+                    al += kStepH;
+                }
             }
             tc::mma_commit(bar);
         }
-        // the rows are prepared: the next block's k, q, rates and beta can come in
-        if (tt >= 0 && !last) issue_kqs(t0 + L);
-        wait_mma();
-        // this block's v has landed (the next block's k, q, rates and beta may be in flight)
-        if (tt >= 0) {
-            if (last) cp_async_wait_group<0>();
-            else cp_async_wait_group<1>();
-        }
+        // while the tensor cores work: phase A of the next block
+        if (!last) phase_a(t0 + L, ra);
+        wait_mma(0);
         if (warp == 0) {
             // A and M to shared memory (lane s < L holds row s of the product)
             float x[L], y[L];
@@ -417,6 +442,8 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
             }
         }
         __syncthreads();                                                            // C2
+        // every thread is done with the next block's staged inputs: the one after it
+        if (tt >= 0 && t0 + 2 * L < p.t_end) issue_kqs(t0 + 2 * L);
 
         if (hf == 1) {
             // u of column j, token by token: u_t = w_t v_t - (S_b^T (a o Dc))_t - sum_{s<t} A_ts u_s
@@ -468,12 +495,12 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
                 bh += kStepU;
                 bl += kStepU;
             }
-            tc::mma_commit(bar);
+            tc::mma_commit(bar + 1);
         }
         {
             // readouts of column j: o_t = (S_b^T (q o Dc))_t + sum_{s<=t} M_ts u_s, with u from
-            // its hi / lo parts in TMEM; warps 0-3 take tokens 0..7, warps 4-7 tokens 8..15 of
-            // the same columns (the same TMEM lanes)
+            // its hi / lo parts in TMEM; warps 0-3 take tokens 0..7 (fewer products: warp 0 also
+            // issues the update), warps 4-7 tokens 8..15 of the same columns (the same TMEM lanes)
             float wq[L], cq[L], u[L], ul[L];
             tc::tmem_ld2x16(tl + G::kDW + L, tl + G::kDWc + L, wq, cq);
             tc::tmem_ld2x16(tl + G::kUHi, tl + G::kULo, u, ul);
@@ -495,7 +522,7 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
                 if (t < n) p.o[((tokb + t0 + t) * p.H + h) * D + jl] = oa + ob;
             }
         }
-        wait_mma();
+        wait_mma(1);
         // S_e = fma(hi + lo, Dc_{L-1}, update): to hi / lo for the next block, or, after the
         // interval's last block, to the row-major buffer
 #pragma unroll 1
@@ -504,7 +531,7 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
             tc::tmem_ld3x16(tl + G::kHi + c0, tl + G::kLo + c0, tl + G::kUpd + c0, hi, lo, up);
 #pragma unroll
             for (int c = 0; c < 16; ++c) {
-                const float x = fmaf(__fadd_rn(hi[c], lo[c]), dall[c0 + c], up[c]);
+                const float x = fmaf(__fadd_rn(hi[c], lo[c]), dall_c[c0 + c], up[c]);
                 if (last) {
                     sbuf[sb_off<D>(c0 + c, jl >> 2) + (jl & 3)] = x;
                 } else {
