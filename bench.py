@@ -68,33 +68,48 @@ def algorithmic_bytes(w, fit_every=1):
     return writeback, alloc, per_head
 
 
-def kernel_sha():
-    """Hash of the sources of the fused write-back kernel (ties an ncu traffic figure to the
-    kernel it was taken on)."""
+# Committed ncu summaries that carry a DRAM traffic figure, per (workload, interval form):
+# the summary and the kernel sources its figure was taken on.
+_CORE = ("qs_wb_row.cuh", "qs_common.cuh", "qs_internal.h")
+TRAFFIC_PROFILES = {
+    ("kda_decode", "token"): ("writeback_kda_decode.md", _CORE),
+    ("kda_prefill", "chunk"): ("writeback_kda_prefill_chunk.md", _CORE + ("qs_chunk.cuh", "qs_tc.cuh")),
+}
+
+
+def kernel_sha(files=_CORE):
+    """Hash of the write-back kernel's sources (ties an ncu traffic figure to the kernel it was
+    taken on)."""
     h = hashlib.sha256()
-    for f in ("qs_wb_row.cuh", "qs_common.cuh", "qs_internal.h"):
+    for f in files:
         with open(os.path.join(ROOT, "paper_2609_30950_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
 
 
-def recorded_traffic(sha):
-    """DRAM bytes per write-back launch from the committed ncu summary, if it was taken on
-    the current kernel sources; else None."""
-    path = os.path.join(ROOT, "profiles", "writeback_kda_decode.md")
+def recorded_traffic(workload, form):
+    """(kernel sha, DRAM bytes per write-back + allocation launch pair) from the committed ncu
+    summary of this workload and interval form, the bytes None unless the summary was taken on
+    the current kernel sources (or there is no summary)."""
+    entry = TRAFFIC_PROFILES.get((workload, form))
+    if entry is None:
+        return kernel_sha(), None
+    name, files = entry
+    sha = kernel_sha(files)
+    path = os.path.join(ROOT, "profiles", name)
     if not os.path.exists(path):
-        return None
+        return sha, None
     vals = {}
     for line in open(path):
         if ":" in line and line.strip().startswith("- "):
             k, v = line.strip()[2:].split(":", 1)
             vals[k.strip()] = v.strip()
     if vals.get("kernel_sha") != sha:
-        return None
+        return sha, None
     try:
-        return float(vals["dram_bytes_per_launch"])
+        return sha, float(vals["dram_bytes_per_launch"])
     except (KeyError, ValueError):
-        return None
+        return sha, None
 
 
 def peaks():
@@ -367,8 +382,7 @@ def main():
     wb_bytes, alloc_bytes, per_head = algorithmic_bytes(w, args.fit_every)
     peak, peak_kind = peaks()
     achieved = (wb_bytes + alloc_bytes) / (per_wb_ms / 1000.0) / 1e9
-    sha = kernel_sha()
-    traffic = recorded_traffic(sha)
+    sha, traffic = recorded_traffic(w.name, args.form)
 
     # end to end through the public API: pinned host inputs -> device, the step, o -> host.
     # The rates go first (the log-decay levels are taken over all tokens of the step); q, k,
