@@ -29,8 +29,8 @@ def _workload(C, bbar, bmin, bmax, T):
                           persistent=1e-3, seed=9000)
 
 
-def _gpu_rel_mse(qs, w, weight_kind, o_ref):
-    cfg = qs.Config.from_workload(w, weight_kind=weight_kind)
+def _gpu_rel_mse(qs, w, weight_kind, o_ref, form=0):
+    cfg = qs.Config.from_workload(w, weight_kind=weight_kind, interval_form=form)
     inp = synth.host_inputs(w)
     d = {k: torch.from_numpy(v).cuda() for k, v in inp.items()}
     X = qs.Inputs(d["q"], d["k"], d["v"], d["s"], None, None, d["beta"], w.T)
@@ -59,14 +59,16 @@ def _gpu_fp32_readouts(qs, w):
 # (C, bbar, bmin, bmax, T, bound on ours / uniform): chunked write-back at a two-bit mean payload
 # (Fig. 1(d), Table 1) and per-token write-back at a four-bit mean (Table 2a); the oracle gives
 # 0.30, 0.31 and 0.21 for the error ratio on these inputs
-CASES = [(64, 2, 1, 8, 512, 0.5), (16, 2, 1, 8, 512, 0.5), (1, 4, 0, 8, 256, 0.4)]
+CASES = [(64, 2, 1, 8, 512, 0.5, 0), (16, 2, 1, 8, 512, 0.5, 0), (1, 4, 0, 8, 256, 0.4, 0),
+         # the chunked form of the write-back intervals (tensor cores)
+         (64, 2, 1, 8, 512, 0.5, 1), (16, 2, 1, 8, 512, 0.5, 1)]
 
 
-@pytest.mark.parametrize("C,bbar,bmin,bmax,T,ratio", CASES)
-def test_allocation_lowers_readout_error(qs, orc, C, bbar, bmin, bmax, T, ratio):
+@pytest.mark.parametrize("C,bbar,bmin,bmax,T,ratio,form", CASES)
+def test_allocation_lowers_readout_error(qs, orc, C, bbar, bmin, bmax, T, ratio, form):
     W = _workload(C, bbar, bmin, bmax, T)
     o_ref = _gpu_fp32_readouts(qs, W)
-    errs = {name: _gpu_rel_mse(qs, W, kind, o_ref)
+    errs = {name: _gpu_rel_mse(qs, W, kind, o_ref, form)
             for name, kind in (("uniform", qs.WEIGHT_UNIFORM), ("ours", qs.WEIGHT_OURS),
                                ("range", qs.WEIGHT_RANGE), ("persistence", qs.WEIGHT_PERSIST))}
     print("relative readout MSE:", ", ".join(f"{k} {v:.4e}" for k, v in errs.items()))
