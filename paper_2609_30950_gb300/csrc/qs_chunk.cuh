@@ -13,9 +13,9 @@
 // The products with S_b (32 columns of S_b^T [a o Dc; q o Dc]^T), the matrices A and M (one
 // product (k / Dc) [a o Dc; q o Dc]^T) and the state update (a rank-16 product) run on the
 // tensor cores; the triangular solve for u and the readouts run on the CUDA cores.  The FP32 state stays in tensor memory (TMEM) as S^T (lane = value column j,
-// column = key row i) for the whole interval, held as its exact split S = hi + lo (hi the top
-// 19 bits, a TF32 number; lo the FP32 remainder).  The products use the 3xTF32 scheme
-// hi*hi + hi*lo + lo*hi (the tensor core truncates its inputs to TF32, so hi is exact).
+// column = key row i) for the whole interval: the FP32 value S and its remainder lo = S - hi
+// below the top 19 bits hi.  The tensor core truncates its FP32 inputs to TF32, so reading S
+// as an operand gives exactly hi; the products use the 3xTF32 scheme hi*hi + hi*lo + lo*hi.
 // The tensor core's FP32 accumulation truncates, so large and small terms are kept apart: the
 // hi*hi and the correction products of S_b^T [..] go to separate accumulators, and the block's
 // update goes to a fresh accumulator that the CUDA cores add to the decayed state with one
@@ -55,7 +55,7 @@ __device__ __forceinline__ void cp_async_wait_group() {
 struct ChunkGeo {
     static constexpr int L = 16;    // tokens per block
     static constexpr int D = 128;   // dk = dv
-    // TMEM columns: S^T as hi / lo, the block's update, the product with S_b (hi*hi part and
+    // TMEM columns: S^T (FP32, read by the products as its TF32 part hi) and lo, the block's update, the product with S_b (hi*hi part and
     // corrections), u^T hi / lo, the product (k / Dc) [a o Dc ; q o Dc]^T that gives A and M
     static constexpr uint32_t kHi = 0, kLo = 128, kUpd = 256, kDW = 384, kDWc = 416, kUHi = 448,
                               kULo = 464, kAM = 480;
@@ -201,17 +201,16 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
     };
     if (tt >= 0 && p.t_begin < p.t_end) issue_kqs(p.t_begin);
 
-    // state in: S^T into TMEM as hi / lo; this thread's lane j, key rows of its half
+    // state in: S^T into TMEM (FP32 and lo); this thread's lane j, key rows of its half
 #pragma unroll 1
     for (int i0 = 64 * hf; i0 < 64 * hf + 64; i0 += 16) {
-        float hi[16], lo[16];
+        float x[16], lo[16];
 #pragma unroll
         for (int c = 0; c < 16; ++c) {
-            const float x = sbuf[sb_off<D>(i0 + c, jl >> 2) + (jl & 3)];
-            hi[c] = tc::tf32_hi(x);
-            lo[c] = __fsub_rn(x, hi[c]);
+            x[c] = sbuf[sb_off<D>(i0 + c, jl >> 2) + (jl & 3)];
+            lo[c] = __fsub_rn(x[c], tc::tf32_hi(x[c]));
         }
-        tc::tmem_st16(tl + G::kHi + i0, hi);
+        tc::tmem_st16(tl + G::kHi + i0, x);
         tc::tmem_st16(tl + G::kLo + i0, lo);
     }
     tc::wait_st();
@@ -523,24 +522,20 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
             }
         }
         wait_mma(1);
-        // S_e = fma(hi + lo, Dc_{L-1}, update): to hi / lo for the next block, or, after the
-        // interval's last block, to the row-major buffer
+        // S_e = fma(S_b, Dc_{L-1}, update): to TMEM (with its lo) for the next block, or, after
+        // the interval's last block, to the row-major buffer
 #pragma unroll 1
         for (int c0 = 64 * hf; c0 < 64 * hf + 64; c0 += 16) {
-            float hi[16], lo[16], up[16];
-            tc::tmem_ld3x16(tl + G::kHi + c0, tl + G::kLo + c0, tl + G::kUpd + c0, hi, lo, up);
+            float x[16], up[16], lo[16];
+            tc::tmem_ld2x16(tl + G::kHi + c0, tl + G::kUpd + c0, x, up);
 #pragma unroll
             for (int c = 0; c < 16; ++c) {
-                const float x = fmaf(__fadd_rn(hi[c], lo[c]), dall_c[c0 + c], up[c]);
-                if (last) {
-                    sbuf[sb_off<D>(c0 + c, jl >> 2) + (jl & 3)] = x;
-                } else {
-                    hi[c] = tc::tf32_hi(x);
-                    lo[c] = __fsub_rn(x, hi[c]);
-                }
+                x[c] = fmaf(x[c], dall_c[c0 + c], up[c]);
+                if (last) sbuf[sb_off<D>(c0 + c, jl >> 2) + (jl & 3)] = x[c];
+                else lo[c] = __fsub_rn(x[c], tc::tf32_hi(x[c]));
             }
             if (!last) {
-                tc::tmem_st16(tl + G::kHi + c0, hi);
+                tc::tmem_st16(tl + G::kHi + c0, x);
                 tc::tmem_st16(tl + G::kLo + c0, lo);
             }
         }
@@ -551,10 +546,10 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
         // no tokens: the state goes back unchanged
 #pragma unroll 1
         for (int i0 = 64 * hf; i0 < 64 * hf + 64; i0 += 16) {
-            float hi[16], lo[16];
-            tc::tmem_ld2x16(tl + G::kHi + i0, tl + G::kLo + i0, hi, lo);
+            float x[16];
+            tc::tmem_ld16(tl + G::kHi + i0, x);
 #pragma unroll
-            for (int c = 0; c < 16; ++c) sbuf[sb_off<D>(i0 + c, jl >> 2) + (jl & 3)] = __fadd_rn(hi[c], lo[c]);
+            for (int c = 0; c < 16; ++c) sbuf[sb_off<D>(i0 + c, jl >> 2) + (jl & 3)] = x[c];
         }
     }
 }
