@@ -46,11 +46,6 @@ __device__ __forceinline__ void cp_async16(void* smem, const void* gmem);
 __device__ __forceinline__ void cp_async4(void* smem, const void* gmem);
 __device__ __forceinline__ void cp_async_commit();
 __device__ __forceinline__ void cp_async_wait_all();
-// Wait until at most N of this thread's cp.async groups are pending (groups complete in order).
-template <int N>
-__device__ __forceinline__ void cp_async_wait_group() {
-    asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
-}
 
 struct ChunkGeo {
     static constexpr int L = 16;    // tokens per block

@@ -46,7 +46,6 @@ __device__ __forceinline__ void fence_after_sync() {
 __device__ __forceinline__ void fence_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
 }
-__device__ __forceinline__ void wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory"); }
 __device__ __forceinline__ void wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;\n" ::: "memory"); }
 
 // ---- registers <-> TMEM, 32 lanes x N columns of 32 bits (lane l of the warp <-> TMEM lane
@@ -83,25 +82,6 @@ __device__ __forceinline__ void tmem_ld2x16(uint32_t ta, uint32_t tb, float (&va
     for (int c = 0; c < 16; ++c) {
         va[c] = __uint_as_float(r[c]);
         vb[c] = __uint_as_float(r[16 + c]);
-    }
-}
-// Three 16-column loads in flight, then one wait (one asm statement, as above).
-__device__ __forceinline__ void tmem_ld3x16(uint32_t ta, uint32_t tb, uint32_t tc_, float (&va)[16], float (&vb)[16],
-                                            float (&vc)[16]) {
-    uint32_t r[48];
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%48];\n"
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%49];\n"
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47}, [%50];\n"
-        "tcgen05.wait::ld.sync.aligned;\n"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47])
-        : "r"(ta), "r"(tb), "r"(tc_)
-        : "memory");
-#pragma unroll
-    for (int c = 0; c < 16; ++c) {
-        va[c] = __uint_as_float(r[c]);
-        vb[c] = __uint_as_float(r[16 + c]);
-        vc[c] = __uint_as_float(r[32 + c]);
     }
 }
 __device__ __forceinline__ void tmem_st16(uint32_t taddr, const float (&v)[16]) {
