@@ -285,6 +285,8 @@ def main():
                          "cores (row unit, 128 x 128, C > 1); auto: the chunked form where it applies")
     ap.add_argument("--T", type=int, default=None, help="tokens per step (default: workload T)")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--e2e-chunk", type=int, default=0,
+                    help="tokens per host-staging chunk of the end-to-end run (default: max(64, C))")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--workload", default=WORKLOAD, choices=sorted(synth.WORKLOADS),
                     help="the paper's layer shape to run (default: KDA decode)")
@@ -401,7 +403,8 @@ def main():
         comp.wait_stream(stream)
         xh = q.Inputs(host_in["q"], host_in["k"], host_in["v"], None if coded else host_in["s"],
                       None, None, host_in.get("beta"), w.T)
-        chunk = max(64, w.C)
+        chunk = args.e2e_chunk if args.e2e_chunk > 0 else max(64, w.C)
+        chunk = -(-chunk // w.C) * w.C   # a multiple of C
 
         def e2e_step():
             if coded:   # the levels are taken over all tokens: the rates go first
