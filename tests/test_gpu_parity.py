@@ -538,15 +538,17 @@ def test_scan_equals_repeated_steps(qs, orc):
 
 
 # ------------------------------------------------------------------ host-staged scan
-@pytest.mark.parametrize("name,chunk", [("kda_decode", 3), ("gdn_decode", 4), ("kda_prefill", 8)])
-def test_scan_host_equals_scan(qs, orc, name, chunk):
+@pytest.mark.parametrize("name,chunk,form", [("kda_decode", 3, 0), ("gdn_decode", 4, 0), ("kda_prefill", 8, 0),
+                                             ("kda_prefill", 8, 1)])
+def test_scan_host_equals_scan(qs, orc, name, chunk, form):
     """qstate_scan_host (inputs copied from pinned host memory chunk by chunk on a second
-    stream) gives qstate_scan's readouts and final state bit for bit."""
+    stream) gives qstate_scan's readouts and final state bit for bit (form 1: both in chunked
+    form)."""
     w = SMALL[name]
     if name == "kda_prefill":
         w = synth.scaled(w, T=2 * w.C + 5)
         chunk = w.C
-    cfgq = qs.Config.from_workload(w)
+    cfgq = qs.Config.from_workload(w, interval_form=form)
     inp = synth.host_inputs(w)
     s_code = s_lut = None
     if w.gate_bits:
