@@ -72,8 +72,8 @@ struct ChunkGeo {
     static constexpr uint32_t oAM = oBuLo + kBu;                  // A and M, L x L each
     static constexpr uint32_t oDall = oAM + 2 * L * L * 4;        // two buffers, by block parity
     static constexpr uint32_t oXch = oDall + 2 * D * 4;          // row preparation: the halves' exchange
-    // mbarriers of the products with S_b and A / M (two arrivals) and of the update (one),
-    // then the TMEM address
+    // mbarriers of the products with S_b and A / M (two arrivals) and of the update (one); the
+    // TMEM address (byte 16), the abort word (byte 20) and the teardown's mbarrier (byte 24)
     static constexpr uint32_t oBar = oXch + 2 * D * 16;
     // one block's token inputs, staged by cp.async: k, q, rates (FP32 per row, per head, or
     // uint8 codes) and beta (three buffers by block index mod 3: block c's solve still reads
@@ -90,8 +90,25 @@ static_assert(ChunkGeo::oBwHi % 16 == 0 && ChunkGeo::oBuHi % 16 == 0 && ChunkGeo
 static_assert(ChunkGeo::oKhLo + (ChunkGeo::D / 8 - 1) * 2 * ChunkGeo::kLboH + ChunkGeo::kLboH + 16 * 128 <=
               ChunkGeo::oBwLo, "aliased operand rows");
 
+__device__ __forceinline__ volatile uint32_t* chunk_abort_word(uint8_t* cb) {
+    return reinterpret_cast<volatile uint32_t*>(cb + ChunkGeo::oBar + 20);
+}
+
+// Wait for phase `parity` of a product mbarrier.  Gives up after kWaitPolls polls and then
+// sets the CTA's abort word; once that word is set every later wait of the CTA gives up at
+// once, so a product that never completes costs one limit, not one per wait.
+__device__ __forceinline__ bool chunk_wait(uint64_t* bar, uint32_t parity, volatile uint32_t* abort) {
+    if (*abort != 0u) return false;
+    for (int it = 0; it < ChunkGeo::kWaitPolls; ++it) {
+        if (tc::mbar_try_wait(bar, parity)) return true;
+        if ((it & 255) == 255 && *abort != 0u) return false;
+    }
+    *abort = 1u;
+    return false;
+}
+
 // Once per CTA: all 512 TMEM columns (the kernel runs one CTA per SM in this form) and the
-// mbarrier of the products.  Returns the TMEM base address.
+// mbarriers of the products.  Returns the TMEM base address.
 __device__ __forceinline__ uint32_t chunk_setup(uint8_t* cb) {
     using G = ChunkGeo;
     const int tid = threadIdx.x;
@@ -104,6 +121,8 @@ __device__ __forceinline__ uint32_t chunk_setup(uint8_t* cb) {
     if (tid == 32) {
         tc::mbar_init(bar, 2);       // products with S_b (thread 0) and for A / M (thread 32)
         tc::mbar_init(bar + 1, 1);   // the update
+        tc::mbar_init(bar + 3, 2);   // teardown after a wait gave up: both issuers' products
+        *chunk_abort_word(cb) = 0u;
         tc::mbar_fence_init();
     }
     tc::fence_before_sync();
@@ -112,10 +131,21 @@ __device__ __forceinline__ uint32_t chunk_setup(uint8_t* cb) {
     return *ta;
 }
 
-__device__ __forceinline__ void chunk_teardown(uint32_t tmem) {
+// Frees the TMEM columns.  If a wait gave up (the abort word, uniform after the barrier),
+// products may still be in flight: both issuing threads commit to the teardown mbarrier and
+// warp 0 waits for it, bounded, before the columns are freed.  Copies in flight are waited
+// for too.
+__device__ __forceinline__ void chunk_teardown(uint32_t tmem, uint8_t* cb) {
+    const int tid = threadIdx.x;
+    cp_async_wait_all();
     tc::fence_before_sync();
     __syncthreads();
-    if (threadIdx.x < 32) {
+    if (*chunk_abort_word(cb) != 0u) {
+        uint64_t* bar = reinterpret_cast<uint64_t*>(cb + ChunkGeo::oBar) + 3;
+        if (tid == 0 || tid == 32) tc::mma_commit(bar);
+        if (tid < 32) tc::mbar_wait(bar, 0u, ChunkGeo::kWaitPolls);
+    }
+    if (tid < 32) {
         tc::fence_after_sync();
         tc::tmem_dealloc(tmem, ChunkGeo::kCols);
     }
@@ -151,8 +181,9 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
     const uint8_t* sc = stg + G::sS;
     const size_t tokb = static_cast<size_t>(b) * p.T;
     // `phase` carries both mbarriers' parities: bit 0 the first's, bit 1 the second's
+    volatile uint32_t* abort = chunk_abort_word(cb);
     auto wait_mma = [&](int which) {
-        if (!tc::mbar_wait(bar + which, (phase >> which) & 1u, G::kWaitPolls)) raise_status(p.status, QS_DEV_TIMEOUT);
+        if (!chunk_wait(bar + which, (phase >> which) & 1u, abort)) raise_status(p.status, QS_DEV_TIMEOUT);
         phase ^= 1u << which;
         tc::fence_after_sync();
     };

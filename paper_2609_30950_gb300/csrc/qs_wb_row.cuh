@@ -904,7 +904,7 @@ __global__ void __launch_bounds__(NW * 32, CHUNK ? 1 : 2) wb_row_kernel(const Wb
             }
         }
     }
-    if constexpr (CHUNK) chunk_teardown(tmem);
+    if constexpr (CHUNK) chunk_teardown(tmem, cb);
 }
 
 template <int DK, int DV, int NW, bool CHUNK = false>
