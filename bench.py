@@ -286,7 +286,8 @@ def main():
     ap.add_argument("--T", type=int, default=None, help="tokens per step (default: workload T)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-chunk", type=int, default=0,
-                    help="tokens per host-staging chunk of the end-to-end run (default: max(64, C))")
+                    help="tokens per host-staging chunk of the end-to-end run (default: 64 when the "
+                         "state is written back every token, else max(256, C))")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--workload", default=WORKLOAD, choices=sorted(synth.WORKLOADS),
                     help="the paper's layer shape to run (default: KDA decode)")
@@ -403,7 +404,10 @@ def main():
         comp.wait_stream(stream)
         xh = q.Inputs(host_in["q"], host_in["k"], host_in["v"], None if coded else host_in["s"],
                       None, None, host_in.get("beta"), w.T)
-        chunk = args.e2e_chunk if args.e2e_chunk > 0 else max(64, w.C)
+        # per-token write-back: 64-token chunks (larger ones measured no faster); write-back
+        # intervals of C > 1 tokens: at least 256 tokens (several intervals per chunk, fewer
+        # staging launches and stream handoffs per write-back)
+        chunk = args.e2e_chunk if args.e2e_chunk > 0 else (64 if w.C == 1 else max(256, w.C))
         chunk = -(-chunk // w.C) * w.C   # a multiple of C
 
         def e2e_step():
