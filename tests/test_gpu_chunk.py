@@ -37,6 +37,9 @@ CASES = {
     # per-head log-quantised rates, row unit
     "gdn_row_coded_c32": (lambda: synth.scaled(synth.WORKLOADS["gdn_decode"], B=2, H=4, T=45, C=32,
                                                unit="row", bmin=1, bmax=8, gate_bits=2), True),
+    # the widest rows (14 bits on average, widths 12..16 allocated): the largest payload
+    # buffer the chunked form's shared memory holds
+    "prefill_wide_c32": (lambda: small("kda_prefill", B=2, H=3, T=70, C=32, bbar=14, bmin=0, bmax=16), False),
     # slow channels that keep their rate over the whole sequence
     "persistent_c64": (lambda: synth.scaled(synth.EXTENSION_WORKLOADS["kda_persistent"], B=2, H=3,
                                             T=130, C=64), True),
@@ -50,7 +53,9 @@ def test_chunked_form_lockstep(qs, orc, case):
     rep = _lockstep(qs, orc, w, log_decay=log_decay, interval_form=CHUNK)
     worst = max(r["rel_o"] for r in rep)
     agree = min(r["code_agree"] for r in rep)
-    print(f"{case}: {len(rep)} write-backs, worst rel readout {worst:.2e}, min code agreement {agree:.6f}")
+    wide = min((r["wide_code_agree"] for r in rep if "wide_code_agree" in r), default=None)
+    print(f"{case}: {len(rep)} write-backs, worst rel readout {worst:.2e}, min code agreement {agree:.6f}"
+          + ("" if wide is None else f", rows wider than 8 bits {wide:.6f}"))
 
 
 def test_chunked_form_refit_schedule(qs, orc):

@@ -602,3 +602,44 @@ def test_scan_host_argument_errors(qs):
         qs.qstate_scan_host(cfgq, A, Bs, xh, X, 0, w.T, 0, oh, o, st, 2, s1, s1)
     with pytest.raises(qs.QstateError):        # chunk not a multiple of C (C = 1: chunk 0)
         qs.qstate_scan_host(cfgq, A, Bs, xh, X, 0, w.T, 0, oh, o, st, 0, s1, torch.cuda.Stream())
+
+
+@pytest.mark.parametrize("form", [0, 1])
+def test_empty_token_range(qs, form):
+    """An empty token range [t, t) is a no-op for qstate_scan and qstate_scan_host (state,
+    statistics and readouts untouched, the state stays in ping) and an error for qstate_step,
+    whose interval holds 1..C tokens; reversed or out-of-range ranges are errors."""
+    w = small("kda_prefill", B=2, H=2, T=40, C=16)
+    cfgq = qs.Config.from_workload(w, interval_form=form)
+    inp = synth.host_inputs(w)
+    X, _ = _dev_inputs(w, inp, qs)
+    A, Bs, st = qs.new_state(cfgq), qs.new_state(cfgq), qs.new_stats(cfgq)
+    qs.qstate_init(cfgq, A, Bs)
+    qs.qstate_scan(cfgq, A, Bs, X, 0, w.C, 0, torch.zeros((w.B, w.T, w.H, w.dv), device="cuda"), st)
+    torch.cuda.synchronize()
+    fields = ("payload", "scales", "widths", "head_off", "fidx")
+    snap = {(n, f): getattr(s, f).clone() for n, s in (("A", A), ("B", Bs)) for f in fields}
+    snap_st = {f: getattr(st, f).clone() for f in ("ema_s", "ema_r", "range")}
+    o = torch.full((w.B, w.T, w.H, w.dv), 3.0, device="cuda")
+    assert not qs.qstate_scan(cfgq, A, Bs, X, 7, 7, 1, o, st)
+    oh = torch.full(o.shape, 3.0).pin_memory()
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    s1.wait_stream(torch.cuda.current_stream())
+    xh = qs.Inputs(*(torch.from_numpy(np.ascontiguousarray(inp[n])).pin_memory() for n in ("q", "k", "v", "s")),
+                   None, None, torch.from_numpy(np.ascontiguousarray(inp["beta"])).pin_memory(), w.T)
+    assert not qs.qstate_scan_host(cfgq, A, Bs, xh, X, 7, 7, 1, oh, o, st, w.C, s1, s2)
+    s1.synchronize()
+    qs.qstate_check()
+    for (n, f), v in snap.items():
+        assert torch.equal(getattr(A if n == "A" else Bs, f), v), (n, f)
+    for f, v in snap_st.items():
+        assert torch.equal(getattr(st, f), v), f
+    assert bool((o == 3.0).all()) and bool((oh == 3.0).all())
+    for t0, t1 in ((7, 7), (9, 8)):
+        with pytest.raises(qs.QstateError) as e:
+            qs.qstate_step(cfgq, A, Bs, X, t0, t1, 1, o, st)
+        assert e.value.code == qs.QSTATE_EINVAL
+    for t0, t1 in ((9, 8), (0, w.T + 1), (-1, 3)):
+        with pytest.raises(qs.QstateError) as e:
+            qs.qstate_scan(cfgq, A, Bs, X, t0, t1, 1, o, st)
+        assert e.value.code == qs.QSTATE_EINVAL

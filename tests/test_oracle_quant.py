@@ -220,3 +220,35 @@ def test_parity_candidate_errors_match_the_oracle(orc):
             _, _, _, sse = orc.quant_group(x, b, with_sse=True)
             got = candidate_sse(x, b, np.max(np.abs(x)))
             assert np.allclose(got, sse, rtol=1e-12, atol=0), (b, got, sse)
+
+
+def test_wide_row_code_criterion(orc):
+    """The parity criterion for rows wider than 8 bits: the oracle quantises a group, then the
+    same group perturbed within half the range tolerance with the oracle's own fitted factor.
+    At 12 and 16 bits some codes change, each by one step and each at a value within the
+    tolerance of a rounding boundary.  At 12 bits the tolerance is 0.02 of a step, so values a
+    quarter step from a boundary are rejected; at 16 bits it spans a third of a step, so there
+    the check reduces to one step; at 8 bits it is a 500th of a step."""
+    from parity import REL_STATS, near_boundary
+    rng = np.random.default_rng(21)
+    x = rng.standard_normal(4096).astype(np.float32)
+    R = float(np.max(np.abs(x)))
+    xp = (x + rng.uniform(-0.5, 0.5, x.size) * REL_STATS * R).astype(np.float32)
+    for b in (12, 16):
+        codes, sc, fidx = orc.quant_group(x, b)
+        D = np.float32(np.array(sc, np.uint16).view(np.float16))
+        codes_p, sc_p, _ = orc.quant_group(xp, b, refit=False, fidx_in=fidx)
+        assert sc_p == sc
+        flip = codes != codes_p
+        assert 0 < flip.sum() < x.size // 10, b
+        assert np.all(np.abs(codes.astype(int) - codes_p.astype(int)) <= 1)
+        assert near_boundary(x[flip], D, R).all(), b
+        tol = REL_STATS * R / D
+        if b == 12:
+            assert tol < 0.05
+            far = ((np.arange(1, 200) + 0.25) * D).astype(np.float32)
+            assert not near_boundary(far, D, R).any()
+        else:
+            assert 0.25 < tol < 0.5
+    D8 = np.float32(np.float16(R / 127))
+    assert REL_STATS * R / D8 < 2e-3
