@@ -454,6 +454,16 @@ def test_quantised_lockstep_chunked_row_kernel(qs, orc, case):
     _lockstep(qs, orc, w, log_decay=log_decay)
 
 
+@pytest.mark.parametrize("name,kw", [("kda_decode", dict(B=2, H=3, T=6)),
+                                     ("gdn_decode", dict(B=2, H=4, T=6)),
+                                     ("kda_prefill", dict(B=1, H=2, T=40, C=16))])
+def test_quantised_lockstep_wide_rows(qs, orc, name, kw):
+    """The widest rows (14 bits on average, widths up to 16) token by token, row unit (KDA)
+    and head unit (Gated DeltaNet); codes of rows wider than 8 bits are checked per code."""
+    w = small(name, bbar=14, bmin=0, bmax=16, gate_bits=0, **kw)
+    _lockstep(qs, orc, w)
+
+
 def test_quantised_lockstep_ragged_chunks(qs, orc):
     w = small("kda_prefill", B=1, H=2, T=37, C=16)
     _lockstep(qs, orc, w)
