@@ -261,7 +261,7 @@ def config_of(w, args):
             "interval_form": getattr(args, "form", "token"),
             "global_batch": w.B * args.gpus, "seq_len": w.T,
             "parallelism": f"dp{args.gpus}",
-            "l2": (f"inputs {input_gb(w):.1f} GB > 129 MB L2: no flush" if input_gb(w) > 0.129
+            "l2": (f"inputs {input_gb(w) * 1e3:.0f} MB > 129 MB L2: no flush" if input_gb(w) > 0.129
                    else f"inputs {input_gb(w) * 1e3:.1f} MB fit in L2 (small case)")}
 
 
