@@ -174,13 +174,25 @@ class ClockSampler:
                 "samples": len(rows)}
 
 
-def cpu_baseline(w, budget_s=12.0):
-    """The oracle as it stands, single-threaded, on a bounded sample of the workload: the
-    log-decay quantiser over the sample's rates (when rates are coded), then per write-back one
-    pass over every head of the sampled batch elements and the allocation.  Returns tokens/s
-    and the sample."""
+def host_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def cpu_baseline(w, budget_s=12.0, parallel=False):
+    """The oracle as it stands on a bounded sample of the workload: the log-decay quantiser over
+    the sample's rates (when rates are coded), then per write-back one pass over every head of
+    the sampled batch elements and the allocation.  Single-threaded (the plain build), or with
+    ``parallel`` the OpenMP timing build, whose threads share out the heads of each write-back
+    over every host core this process may use (same arithmetic).  Returns tokens/s and the
+    sample."""
     import numpy as np
     from oracle import oracle as orc
+    cores = host_cores() if parallel else 1
+    if parallel:
+        os.environ["OMP_NUM_THREADS"] = str(cores)
     nb, nt = 4, max(64, w.C)
     sub = synth.scaled(w, B=nb)
     cfg = orc.Cfg.from_workload(sub)
@@ -196,17 +208,32 @@ def cpu_baseline(w, budget_s=12.0):
     ms, mr, R = (np.zeros(cfg.units * nb, np.float32) for _ in range(3))
     tokens = 0
     for wi, t in enumerate(range(0, nt, w.C)):
-        orc.step(cfg, src, dst, inp, t, t + w.C, wi, o, ms, mr, R, codes, lut)
+        orc.step(cfg, src, dst, inp, t, t + w.C, wi, o, ms, mr, R, codes, lut, parallel=parallel)
         src.widths[:], src.head_off[:] = orc.alloc(cfg, ms, mr, R)
         src, dst = dst, src
         tokens += nb * w.C
         if time.perf_counter() - t0 > budget_s:
             break
     el = time.perf_counter() - t0
-    return tokens / el, dict(cores=1, sample=f"{nb} batch elements x {tokens // nb} tokens x "
-                                             f"{w.H} heads, single thread (input synthesis "
-                                             f"{gen_s:.1f}s excluded)",
+    how = f"OpenMP over the heads, {cores} threads" if parallel else "single thread"
+    return tokens / el, dict(cores=cores, sample=f"{nb} batch elements x {tokens // nb} tokens x "
+                                                 f"{w.H} heads, {how} (input synthesis "
+                                                 f"{gen_s:.1f}s excluded)",
                              seconds=el)
+
+
+def cpu_baselines(w, budget_s):
+    """The oracle on all host cores (the reported baseline) and single-threaded beside it."""
+    one, info1 = cpu_baseline(w, budget_s)
+    try:
+        par, info = cpu_baseline(w, budget_s, parallel=True)
+    except Exception as e:   # no OpenMP compiler: the single-thread figure only
+        return one, info1, {"value": one, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                            "sample": info1["sample"], "all_cores": f"unavailable: {e}"}
+    return par, info, {"value": par, "unit": "tokens/s", "cores": info["cores"], "kind": "oracle",
+                       "sample": info["sample"],
+                       "single_thread": {"value": one, "unit": "tokens/s", "cores": 1,
+                                         "sample": info1["sample"]}}
 
 
 def run_reference(args, w):
@@ -215,7 +242,8 @@ def run_reference(args, w):
         return
     vals = []
     for i in range(args.warmup + args.steps):
-        v, info = cpu_baseline(w, budget_s=max(3.0, 40.0 / max(1, args.steps + args.warmup)))
+        v, info = cpu_baseline(w, budget_s=max(3.0, 40.0 / max(1, args.steps + args.warmup)),
+                               parallel=True)
         if i >= args.warmup:
             vals.append(v)
     value = statistics.median(vals)
@@ -446,9 +474,7 @@ def main():
         return
     cpu = None
     if not args.no_cpu:
-        v, info = cpu_baseline(w)
-        cpu = {"value": v, "unit": "tokens/s", "cores": info["cores"], "kind": "oracle",
-               "sample": info["sample"]}
+        _, _, cpu = cpu_baselines(w, 10.0)
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,

@@ -41,7 +41,10 @@ extern "C" {
 #define QSTATE_EINVAL 1  /* invalid argument or configuration                                */
 #define QSTATE_EBUDGET 2 /* N*bmin > N*bbar or N*bbar > N*bmax: the layer budget is unmeetable */
 #define QSTATE_ECUDA 3   /* a CUDA runtime call failed (message in qstate_last_error)          */
-#define QSTATE_EDEVICE 4 /* a kernel reported an inconsistent device-side layout or input      */
+#define QSTATE_EDEVICE 4 /* a kernel reported an inconsistent device-side layout or input, or
+                            the device was marked unusable (see qstate_check)                 */
+#define QSTATE_ETIMEOUT 5 /* a bounded device-side wait gave up (chunked form: a tensor-core
+                             product did not signal completion within the wait limit)         */
 
 /* ---- configuration enums ---------------------------------------------------------------- */
 #define QSTATE_DECAY_ROW 0   /* one rate per key row (KDA, Sec. 1)                            */
@@ -268,8 +271,23 @@ int qstate_scan_host(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong,
 int qstate_scan_fp32(const qstate_cfg* cfg, float* S, const qstate_inputs* x, int32_t t_begin,
                      int32_t t_end, float* o, void* stream);
 
-/* Synchronise `stream`, read and clear the device status word: QSTATE_OK or QSTATE_EDEVICE. */
+/* Synchronise `stream`, read and clear the device status word.  QSTATE_OK; QSTATE_ETIMEOUT if a
+ * bounded wait of the chunked form gave up (the call's results are not valid; the kernel still
+ * waited for its products before freeing tensor memory, so later calls are unaffected);
+ * otherwise QSTATE_EDEVICE with the reasons in qstate_last_error().  If even that last wait
+ * gave up, tensor memory may have been freed under products in flight: the device is then
+ * marked unusable and every later call that launches work on it (and qstate_check) returns
+ * QSTATE_EDEVICE for the rest of the process. */
 int qstate_check(void* stream);
+
+/* Limit, in polls of the mbarrier, of the chunked form's waits for its tensor-core products in
+ * the calls that follow (process-wide; read when a call is enqueued).  polls >= 0 sets it; 0
+ * gives up at the first wait without polling (the products still complete, the results of
+ * that call are invalid and qstate_check reports QSTATE_ETIMEOUT): a way to exercise the
+ * timeout path without a faulty kernel.  polls < 0 restores the default (2^24 polls, far
+ * beyond any product's latency).  The wait before freeing tensor memory always uses the
+ * default.  Always QSTATE_OK.  Not part of the paper's method: a diagnostic of this library. */
+int qstate_set_wait_limit(int32_t polls);
 
 /* Message for the last failure on this host thread ("" if none).  Valid until the next call. */
 const char* qstate_last_error(void);

@@ -21,17 +21,32 @@ import numpy as np
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "qstate_oracle.c")
 _LIB = os.path.join(_HERE, "_build", "liborc.so")
+# timing build: the same source with a write-back's heads shared out over OpenMP threads
+# (identical arithmetic per head); the checker is always the plain single-thread build
+_LIB_OMP = os.path.join(_HERE, "_build", "liborc_omp.so")
+_FLAGS = ["-std=c11", "-O2", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared"]
+
+
+def _gcc(out, extra):
+    if not os.path.exists(out) or os.path.getmtime(out) < os.path.getmtime(_SRC):
+        os.makedirs(os.path.dirname(out), exist_ok=True)
+        tmp = out + f".{os.getpid()}.tmp"
+        subprocess.check_call(["gcc", *_FLAGS, *extra, "-o", tmp, _SRC, "-lm"])
+        os.replace(tmp, out)
+    return out
 
 
 def build(force: bool = False) -> str:
     """Compile the oracle with gcc (no FMA contraction, no fast-math)."""
-    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
-        os.makedirs(os.path.dirname(_LIB), exist_ok=True)
-        tmp = _LIB + f".{os.getpid()}.tmp"
-        subprocess.check_call(["gcc", "-std=c11", "-O2", "-ffp-contract=off", "-fno-fast-math",
-                               "-fPIC", "-shared", "-o", tmp, _SRC, "-lm"])
-        os.replace(tmp, _LIB)
-    return _LIB
+    if force and os.path.exists(_LIB):
+        os.remove(_LIB)
+    return _gcc(_LIB, [])
+
+
+def build_parallel() -> str:
+    """Compile the OpenMP timing build (heads of a write-back in parallel; used only to time
+    the oracle on all host cores)."""
+    return _gcc(_LIB_OMP, ["-fopenmp", "-DORC_OPENMP"])
 
 
 class OrcCfg(ct.Structure):
@@ -93,39 +108,49 @@ class Cfg:
 
 
 _lib = None
+_lib_par = None
 
 
-def lib():
-    global _lib
+def lib(parallel: bool = False):
+    """The plain build (the checker), or with ``parallel`` the OpenMP timing build."""
+    global _lib, _lib_par
+    if parallel:
+        if _lib_par is None:
+            _lib_par = _declare(ct.CDLL(build_parallel()))
+        return _lib_par
     if _lib is None:
-        _lib = ct.CDLL(build())
-        P = ct.c_void_p
-        L = _lib
-        L.orc_bits_per_element.restype = ct.c_double
-        L.orc_bits_per_element.argtypes = [ct.POINTER(OrcCfg)]
-        L.orc_expm1_series.restype = ct.c_float
-        L.orc_expm1_series.argtypes = [ct.c_float]
-        L.orc_recur_f32.argtypes = [ct.c_int] * 3 + [P] * 8
-        L.orc_recur_f64.argtypes = [ct.c_int] * 3 + [P] * 8
-        L.orc_quant_group.argtypes = [P, ct.c_int, ct.c_int, ct.c_int, ct.c_int, ct.c_int,
-                                      P, P, P, P]
-        L.orc_dequant_group.argtypes = [P, ct.c_int, ct.c_int, ct.c_uint16, P, ct.c_int]
-        L.orc_pack_codes.argtypes = [P, ct.c_int, ct.c_int, P]
-        L.orc_unpack_codes.argtypes = [P, ct.c_int, ct.c_int, P]
-        L.orc_region_bytes.restype = ct.c_long
-        L.orc_region_bytes.argtypes = [ct.POINTER(OrcCfg)]
-        L.orc_pack.argtypes = [ct.POINTER(OrcCfg)] + [P] * 7
-        L.orc_unpack.argtypes = [ct.POINTER(OrcCfg)] + [P] * 5
-        L.orc_weights.argtypes = [ct.POINTER(OrcCfg), ct.c_int, P, P, P, P]
-        L.orc_shuffle.argtypes = [ct.c_int, ct.POINTER(ct.c_int), ct.POINTER(ct.c_int)]
-        L.orc_alloc_from_weights.argtypes = [ct.c_int, P, ct.c_int, ct.c_int, ct.c_long,
-                                             ct.c_int, ct.c_int, P]
-        L.orc_alloc.argtypes = [ct.POINTER(OrcCfg), P, P, P, P, P]
-        L.orc_init_widths.argtypes = [ct.POINTER(OrcCfg), P, P]
-        L.orc_quant_decay.argtypes = [ct.c_long, ct.c_int, P, ct.c_int, P, P, P]
-        L.orc_step.argtypes = ([ct.POINTER(OrcCfg)] + [P] * 10 + [ct.c_int] * 4 + [P] * 14)
-        L.orc_step_current.argtypes = ([ct.POINTER(OrcCfg)] + [P] * 10 + [ct.c_int] * 4 + [P] * 14)
+        _lib = _declare(ct.CDLL(build()))
     return _lib
+
+
+def _declare(L):
+    """Argument and result types of the exported functions."""
+    P = ct.c_void_p
+    L.orc_bits_per_element.restype = ct.c_double
+    L.orc_bits_per_element.argtypes = [ct.POINTER(OrcCfg)]
+    L.orc_expm1_series.restype = ct.c_float
+    L.orc_expm1_series.argtypes = [ct.c_float]
+    L.orc_recur_f32.argtypes = [ct.c_int] * 3 + [P] * 8
+    L.orc_recur_f64.argtypes = [ct.c_int] * 3 + [P] * 8
+    L.orc_quant_group.argtypes = [P, ct.c_int, ct.c_int, ct.c_int, ct.c_int, ct.c_int,
+                                  P, P, P, P]
+    L.orc_dequant_group.argtypes = [P, ct.c_int, ct.c_int, ct.c_uint16, P, ct.c_int]
+    L.orc_pack_codes.argtypes = [P, ct.c_int, ct.c_int, P]
+    L.orc_unpack_codes.argtypes = [P, ct.c_int, ct.c_int, P]
+    L.orc_region_bytes.restype = ct.c_long
+    L.orc_region_bytes.argtypes = [ct.POINTER(OrcCfg)]
+    L.orc_pack.argtypes = [ct.POINTER(OrcCfg)] + [P] * 7
+    L.orc_unpack.argtypes = [ct.POINTER(OrcCfg)] + [P] * 5
+    L.orc_weights.argtypes = [ct.POINTER(OrcCfg), ct.c_int, P, P, P, P]
+    L.orc_shuffle.argtypes = [ct.c_int, ct.POINTER(ct.c_int), ct.POINTER(ct.c_int)]
+    L.orc_alloc_from_weights.argtypes = [ct.c_int, P, ct.c_int, ct.c_int, ct.c_long,
+                                         ct.c_int, ct.c_int, P]
+    L.orc_alloc.argtypes = [ct.POINTER(OrcCfg), P, P, P, P, P]
+    L.orc_init_widths.argtypes = [ct.POINTER(OrcCfg), P, P]
+    L.orc_quant_decay.argtypes = [ct.c_long, ct.c_int, P, ct.c_int, P, P, P]
+    L.orc_step.argtypes = ([ct.POINTER(OrcCfg)] + [P] * 10 + [ct.c_int] * 4 + [P] * 14)
+    L.orc_step_current.argtypes = ([ct.POINTER(OrcCfg)] + [P] * 10 + [ct.c_int] * 4 + [P] * 14)
+    return L
 
 
 def _p(a):
@@ -358,10 +383,11 @@ def init_state(cfg: Cfg):
 
 
 def step(cfg: Cfg, src: Buf, dst: Buf, inp: dict, t_begin, t_end, w_index, o, ema_s, ema_r,
-         rng, s_code=None, s_lut=None, want_x=False):
+         rng, s_code=None, s_lut=None, want_x=False, parallel=False):
     """Run tokens [t_begin, t_end) from ``src`` into ``dst`` (whose widths/offsets are the
     target).  ``inp`` holds the full (B, T, H, .) inputs; ``o`` (B, T, H, dv) is written.
-    Returns the FP32 pre-quantisation state if ``want_x``."""
+    Returns the FP32 pre-quantisation state if ``want_x``.  ``parallel`` runs the OpenMP
+    timing build (same results)."""
     T = inp["q"].shape[1]
     c = cfg.c()
     x = np.zeros((cfg.B, cfg.H, cfg.dk, cfg.dv), np.float32) if want_x else None
@@ -372,7 +398,7 @@ def step(cfg: Cfg, src: Buf, dst: Buf, inp: dict, t_begin, t_end, w_index, o, em
     w_in = _c(inp["w"], np.float32) if "w" in inp else None
     sc = None if s_code is None else _c(s_code, np.uint8)
     sl = None if s_lut is None else _c(s_lut, np.float32)
-    fn = lib().orc_step_current if cfg.alloc_mode == 1 else lib().orc_step
+    fn = lib().orc_step_current if cfg.alloc_mode == 1 else lib(parallel).orc_step
     rc = fn(ct.byref(c), _p(src.payload), _p(src.scales), _p(src.widths),
                         _p(src.head_off), _p(src.fidx), _p(dst.payload), _p(dst.scales),
                         _p(dst.widths), _p(dst.head_off), _p(dst.fidx), T, t_begin, t_end,

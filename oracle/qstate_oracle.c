@@ -724,12 +724,24 @@ int orc_step(const orc_cfg* c, const uint8_t* pay_in, const uint16_t* sc_in, con
     if (rb < 0 || !layout_ok(c, w_in, off_in) || !layout_ok(c, w_out, off_out)) return ORC_EINVAL;
     if (c->erase_kind == 2 && (!a_tok || !w_tok)) return ORC_EINVAL;
     float alpha = 2.0f / (c->ema_span + 1.0f);
+    memset(pay_out, 0, (size_t)c->B * (size_t)rb);
+    /* Heads are independent within a write-back (each writes only its own bytes, scales,
+     * statistics and readouts), so the timing build (ORC_OPENMP) shares them out over threads;
+     * every head's arithmetic is the same sequential code either way. */
+    const int nbh = c->B * H;
+#ifdef ORC_OPENMP
+#pragma omp parallel
+#endif
+    {
     float* X = (float*)malloc(sizeof(float) * (size_t)dk * dv);
     float* d = (float*)malloc(sizeof(float) * dk);
     float* p = (float*)malloc(sizeof(float) * dv);
-    for (int b = 0; b < c->B; b++) {
-        memset(pay_out + (size_t)b * rb, 0, (size_t)rb);
-        for (int h = 0; h < H; h++) {
+#ifdef ORC_OPENMP
+#pragma omp for schedule(dynamic, 1)
+#endif
+    for (int bh = 0; bh < nbh; bh++) {
+        const int b = bh / H, h = bh % H;
+        {
             unpack_head(c, b, h, pay_in, sc_in, w_in, off_in, X);
             for (int t = t_begin; t < t_end; t++) {
                 size_t tok = ((size_t)b * T + t) * H + h;
@@ -825,6 +837,7 @@ int orc_step(const orc_cfg* c, const uint8_t* pay_in, const uint16_t* sc_in, con
     free(X);
     free(d);
     free(p);
+    }
     return ORC_OK;
 }
 

@@ -13,7 +13,7 @@ from dataclasses import dataclass, field
 
 from . import build as _build
 
-QSTATE_OK, QSTATE_EINVAL, QSTATE_EBUDGET, QSTATE_ECUDA, QSTATE_EDEVICE = range(5)
+QSTATE_OK, QSTATE_EINVAL, QSTATE_EBUDGET, QSTATE_ECUDA, QSTATE_EDEVICE, QSTATE_ETIMEOUT = range(6)
 DECAY_ROW, DECAY_HEAD = 0, 1
 ERASE_DELTA, ERASE_NONE, ERASE_GENERAL = 0, 1, 2
 ALLOC_LAGGED, ALLOC_CURRENT = 0, 1
@@ -60,7 +60,7 @@ EXPORTS = ["qstate_validate", "qstate_region_bytes", "qstate_units", "qstate_sca
            "qstate_bits_per_element", "qstate_init", "qstate_alloc_bits", "qstate_pack",
            "qstate_unpack", "qstate_quant_decay", "qstate_quant_decay_noalloc", "qstate_step",
            "qstate_scan", "qstate_scan_host",
-           "qstate_scan_fp32", "qstate_check", "qstate_last_error"]
+           "qstate_scan_fp32", "qstate_check", "qstate_set_wait_limit", "qstate_last_error"]
 
 _lib = None
 
@@ -106,6 +106,7 @@ def load(path: str | None = None, build_if_missing: bool = False):
                                    ct.POINTER(_Stats), ct.c_int32, ct.POINTER(ct.c_int32), P, P]
     L.qstate_scan_fp32.argtypes = [PC, P, ct.POINTER(_Inputs), ct.c_int32, ct.c_int32, P, P]
     L.qstate_check.argtypes = [P]
+    L.qstate_set_wait_limit.argtypes = [ct.c_int32]
     L.qstate_last_error.restype = ct.c_char_p
     for name in EXPORTS:
         if name not in ("qstate_region_bytes", "qstate_units", "qstate_scale_groups",
@@ -353,3 +354,9 @@ def qstate_scan_fp32(cfg: Config, S, x: Inputs, t_begin: int, t_end: int, o, str
 
 def qstate_check(stream=None) -> None:
     _check(_lib_or_raise().qstate_check(_stream(stream)))
+
+
+def qstate_set_wait_limit(polls: int) -> None:
+    """Limit of the chunked form's waits for its tensor-core products in later calls (polls;
+    0 gives up at once, negative restores the default)."""
+    _check(_lib_or_raise().qstate_set_wait_limit(int(polls)))

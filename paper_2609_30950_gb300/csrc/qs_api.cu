@@ -1,5 +1,8 @@
 // qs_api.cu -- the C ABI of libqstate (declared in include/qstate.h): host-side validation,
 // error reporting and kernel dispatch.
+#include <cuda.h>   // driver types only (CUcontext); entry points come through the runtime
+
+#include <atomic>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -15,6 +18,49 @@ cudaError_t launch_wb_row_128x128(const qstate_cfg&, const StepParams&, cudaStre
 cudaError_t launch_wb_row_128x64(const qstate_cfg&, const StepParams&, cudaStream_t);
 cudaError_t launch_wb_row_64x64(const qstate_cfg&, const StepParams&, cudaStream_t);
 cudaError_t launch_wb_chunk_128x128(const qstate_cfg&, const StepParams&, cudaStream_t);
+
+// Streaming multiprocessors of the current device, queried once per device.
+int device_sm_count() {
+    static std::atomic<int> cache[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+    int n = cache[dev].load();
+    if (n <= 0) {
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) return 1;
+        cache[dev].store(n);
+    }
+    return n;
+}
+
+// Identity of the calling thread's current CUDA context (cuCtxGetId), fetched through the
+// runtime so that the library does not link the driver library.  A context that is destroyed
+// and created again (cudaDeviceReset, a primary-context reset by a host framework) gets a new
+// identity, and with it the module holding this library's device variables may be loaded at
+// new addresses: host-side caches of those addresses are keyed on it.  False if there is no
+// current context or the driver lacks the call.
+bool current_context_id(unsigned long long* id) {
+    using GetCurrent = CUresult (*)(CUcontext*);
+    using GetId = CUresult (*)(CUcontext, unsigned long long*);
+    static GetCurrent get_current = nullptr;
+    static GetId get_id = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_current = reinterpret_cast<GetCurrent>(f);
+        f = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_id = reinterpret_cast<GetId>(f);
+    });
+    if (!get_current || !get_id) return false;
+    CUcontext ctx = nullptr;
+    if (get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr) return false;
+    return get_id(ctx, id) == CUDA_SUCCESS;
+}
+
 }  // namespace qs
 
 using namespace qs;
@@ -40,21 +86,49 @@ int cuda_fail(cudaError_t e, const char* what) {
 
 constexpr int kMaxDevices = 64;
 std::mutex g_mu;
+// per device: the status word's address and the context it was looked up in
 int* g_status_addr[kMaxDevices] = {};
+unsigned long long g_status_ctx[kMaxDevices] = {};
+// Devices on which a chunked-form teardown wait gave up (QS_DEV_TEARDOWN): tensor memory may
+// have been freed under products still in flight, so later results could not be trusted and
+// every launching call is refused for the rest of the process.
+std::atomic<bool> g_unusable[kMaxDevices] = {};
+// Limit of the chunked form's mbarrier waits for the following launches (qstate_set_wait_limit).
+std::atomic<int> g_wait_polls{kDefaultWaitPolls};
 
-// Address of the status word on the current device, looked up once per device.
-int* status_word(cudaError_t* err) {
+// Address of the status word on the current device, looked up once per device and context
+// (again whenever the context's identity is unknown or has changed).
+int* status_word(cudaError_t* err, int* dev_out = nullptr) {
     int dev = 0;
     *err = cudaGetDevice(&dev);
     if (*err != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+    if (dev_out) *dev_out = dev;
     std::lock_guard<std::mutex> lock(g_mu);
-    if (!g_status_addr[dev]) {
+    unsigned long long ctx = 0;
+    const bool known = current_context_id(&ctx);
+    if (!g_status_addr[dev] || !known || ctx != g_status_ctx[dev]) {
         void* p = nullptr;
         *err = cudaGetSymbolAddress(&p, qs_status_word);
         if (*err != cudaSuccess) return nullptr;
         g_status_addr[dev] = static_cast<int*>(p);
+        // the lookup makes the context current if it was not yet
+        g_status_ctx[dev] = current_context_id(&ctx) ? ctx : 0ull;
     }
     return g_status_addr[dev];
+}
+
+// The status word of the current device for a call that launches work; refused (EDEVICE) once
+// the device has been marked unusable.
+int acquire_status(int** out) {
+    cudaError_t e = cudaSuccess;
+    int dev = -1;
+    int* p = status_word(&e, &dev);
+    if (!p) return cuda_fail(e, "status word");
+    if (g_unusable[dev].load())
+        return fail(QSTATE_EDEVICE, "device %d is marked unusable: a tensor-core teardown wait gave up "
+                    "earlier in this process", dev);
+    *out = p;
+    return QSTATE_OK;
 }
 
 long long units_of(const qstate_cfg* c) {
@@ -166,6 +240,7 @@ StepParams base_params(const qstate_cfg* c, int* status) {
     p.group_heads = c->group_heads;
     p.region_bytes = region_of(c);
     p.alpha = 2.0f / (c->ema_span + 1.0f);
+    p.wait_polls = g_wait_polls.load();
     p.status = status;
     return p;
 }
@@ -288,9 +363,9 @@ int qstate_init(const qstate_cfg* cfg, qstate_buf* a, qstate_buf* b, void* strea
     if (rc) return rc;
     if (!buf_ok(a) || !buf_ok(b)) return fail(QSTATE_EINVAL, "null buffer pointer");
     cudaStream_t st = static_cast<cudaStream_t>(stream);
+    int* status = nullptr;
+    if ((rc = acquire_status(&status))) return rc;
     cudaError_t e;
-    int* status = status_word(&e);
-    if (!status) return cuda_fail(e, "status word");
     rc = run_alloc(cfg, nullptr, nullptr, nullptr, 1, a->widths, a->head_off, status, st);
     if (rc) return rc;
     const size_t nw = static_cast<size_t>(cfg->B) * units_of(cfg);
@@ -317,9 +392,9 @@ int qstate_alloc_bits(const qstate_cfg* cfg, const qstate_stats* stats, uint8_t*
     if (!stats || !stats->ema_s || !stats->ema_r || !widths_out || !head_off_out ||
         (cfg->unit_kind == QSTATE_UNIT_ROW && !stats->range))
         return fail(QSTATE_EINVAL, "null pointer");
+    int* status = nullptr;
+    if ((rc = acquire_status(&status))) return rc;
     cudaError_t e;
-    int* status = status_word(&e);
-    if (!status) return cuda_fail(e, "status word");
     return run_alloc(cfg, stats->ema_s, stats->ema_r, stats->range, 0, widths_out, head_off_out,
                      status, static_cast<cudaStream_t>(stream));
 }
@@ -328,9 +403,9 @@ int qstate_pack(const qstate_cfg* cfg, const float* S, qstate_buf* out, float* r
     int rc = validate(cfg);
     if (rc) return rc;
     if (!S || !buf_ok(out)) return fail(QSTATE_EINVAL, "null pointer");
+    int* status = nullptr;
+    if ((rc = acquire_status(&status))) return rc;
     cudaError_t e;
-    int* status = status_word(&e);
-    if (!status) return cuda_fail(e, "status word");
     StepParams p = base_params(cfg, status);
     p.fit_every = 1;
     p.dense_in = S;
@@ -348,9 +423,9 @@ int qstate_unpack(const qstate_cfg* cfg, const qstate_buf* in, float* S_out, voi
     int rc = validate(cfg);
     if (rc) return rc;
     if (!S_out || !buf_ok(in)) return fail(QSTATE_EINVAL, "null pointer");
+    int* status = nullptr;
+    if ((rc = acquire_status(&status))) return rc;
     cudaError_t e;
-    int* status = status_word(&e);
-    if (!status) return cuda_fail(e, "status word");
     StepParams p = base_params(cfg, status);
     p.in_payload = in->payload;
     p.in_scales = in->scales;
@@ -368,9 +443,9 @@ int qstate_quant_decay(const qstate_cfg* cfg, const float* s, int32_t T, uint8_t
     if (rc) return rc;
     if (cfg->gate_bits < 1) return fail(QSTATE_EINVAL, "gate_bits must be >= 1");
     if (!s || !code_out || !lut_out || !thr_out || T < 1) return fail(QSTATE_EINVAL, "null pointer or T < 1");
+    int* status = nullptr;
+    if ((rc = acquire_status(&status))) return rc;
     cudaError_t e;
-    int* status = status_word(&e);
-    if (!status) return cuda_fail(e, "status word");
     const int nchan = cfg->decay_kind == QSTATE_DECAY_ROW ? cfg->H * cfg->dk : cfg->H;
     const long long count = static_cast<long long>(cfg->B) * T;
     e = launch_quant_decay(s, count, nchan, cfg->gate_bits, code_out, lut_out, thr_out, status,
@@ -391,9 +466,9 @@ int qstate_quant_decay_noalloc(const qstate_cfg* cfg, const float* s, int32_t T,
                     "qstate_quant_decay_noalloc: %lld thresholds (%d channels x %d) exceed the "
                     "built-in scratch of %lld; use qstate_quant_decay with a caller buffer",
                     need, nchan, (1 << cfg->gate_bits) - 1, quant_decay_scratch_capacity());
+    int* status = nullptr;
+    if ((rc = acquire_status(&status))) return rc;
     cudaError_t e;
-    int* status = status_word(&e);
-    if (!status) return cuda_fail(e, "status word");
     float* thr = nullptr;
     e = quant_decay_scratch(&thr);
     if (e != cudaSuccess) return cuda_fail(e, "threshold scratch lookup");
@@ -416,9 +491,9 @@ int qstate_step(const qstate_cfg* cfg, qstate_buf* in, qstate_buf* out, const qs
         return fail(QSTATE_EINVAL, "a write-back interval holds 1..C tokens");
     if (x->s_code && cfg->gate_bits < 1) return fail(QSTATE_EINVAL, "s_code needs gate_bits");
     cudaStream_t st = static_cast<cudaStream_t>(stream);
+    int* status = nullptr;
+    if ((rc = acquire_status(&status))) return rc;
     cudaError_t e;
-    int* status = status_word(&e);
-    if (!status) return cuda_fail(e, "status word");
     StepParams p = base_params(cfg, status);
     set_inputs(p, x);
     p.t_begin = t_begin;
@@ -519,7 +594,7 @@ int qstate_scan_host(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong,
         const bool a16 = per % 16 == 0 && (reinterpret_cast<uintptr_t>(dst) & 15) == 0 &&
                          (reinterpret_cast<uintptr_t>(src) & 15) == 0;
         if (a16) {
-            stage_tokens_kernel<<<2 * 152, 128, 0, ts>>>(static_cast<uint4*>(dst), static_cast<const uint4*>(src),
+            stage_tokens_kernel<<<2 * device_sm_count(), 128, 0, ts>>>(static_cast<uint4*>(dst), static_cast<const uint4*>(src),
                                                         B, static_cast<long long>(pitch / 16),
                                                         static_cast<long long>(off / 16),
                                                         static_cast<long long>(width / 16));
@@ -590,9 +665,9 @@ int qstate_scan_fp32(const qstate_cfg* cfg, float* S, const qstate_inputs* x, in
     if (rc) return rc;
     if (!S) return fail(QSTATE_EINVAL, "S is NULL");
     if ((rc = check_inputs(cfg, x, t_begin, t_end, o))) return rc;
+    int* status = nullptr;
+    if ((rc = acquire_status(&status))) return rc;
     cudaError_t e;
-    int* status = status_word(&e);
-    if (!status) return cuda_fail(e, "status word");
     StepParams p = base_params(cfg, status);
     set_inputs(p, x);
     p.dense_in = S;
@@ -611,7 +686,8 @@ int qstate_check(void* stream) {
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     cudaError_t e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
-    int* status = status_word(&e);
+    int dev = -1;
+    int* status = status_word(&e, &dev);
     if (!status) return cuda_fail(e, "status word");
     int v = 0;
     e = cudaMemcpy(&v, status, sizeof(int), cudaMemcpyDeviceToHost);
@@ -620,12 +696,24 @@ int qstate_check(void* stream) {
         const int zero = 0;
         e = cudaMemcpy(status, &zero, sizeof(int), cudaMemcpyHostToDevice);
         if (e != cudaSuccess) return cuda_fail(e, "status clear");
-        return fail(QSTATE_EDEVICE, "device status 0x%x:%s%s%s%s", v,
+        if (v & QS_DEV_TEARDOWN) g_unusable[dev].store(true);
+        const int code = (v & QS_DEV_TEARDOWN) ? QSTATE_EDEVICE
+                         : (v & QS_DEV_TIMEOUT) ? QSTATE_ETIMEOUT : QSTATE_EDEVICE;
+        return fail(code, "device status 0x%x:%s%s%s%s%s", v,
                     (v & QS_DEV_LAYOUT) ? " inconsistent widths/offsets" : "",
                     (v & QS_DEV_RATE) ? " decay rate not positive/finite" : "",
                     (v & QS_DEV_TIMEOUT) ? " tensor-core product timed out" : "",
-                    (v & QS_DEV_CHUNK) ? " decay over a 16-token block beyond the chunked form's range" : "");
+                    (v & QS_DEV_CHUNK) ? " decay over a 16-token block beyond the chunked form's range" : "",
+                    (v & QS_DEV_TEARDOWN) ? " the wait before freeing tensor memory gave up too: device marked unusable" : "");
     }
+    if (g_unusable[dev].load())
+        return fail(QSTATE_EDEVICE, "device %d is marked unusable: a tensor-core teardown wait gave up "
+                    "earlier in this process", dev);
+    return QSTATE_OK;
+}
+
+int qstate_set_wait_limit(int32_t polls) {
+    g_wait_polls.store(polls < 0 ? kDefaultWaitPolls : polls);
     return QSTATE_OK;
 }
 

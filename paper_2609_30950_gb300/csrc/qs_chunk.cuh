@@ -17,7 +17,8 @@
 // below the top 19 bits hi.  The tensor core truncates its FP32 inputs to TF32, so reading S
 // as an operand gives exactly hi; the products use the 3xTF32 scheme hi*hi + hi*lo + lo*hi.
 // The tensor core's FP32 accumulation truncates, so large and small terms are kept apart: the
-// hi*hi and the correction products of S_b^T [..] go to separate accumulators, and the block's
+// hi*hi and the correction products of S_b^T [..] and of A and M go to separate accumulators
+// (summed with one rounding when read), and the block's
 // update goes to a fresh accumulator that the CUDA cores add to the decayed state with one
 // rounding, S_e = fma(hi + lo, Dc_{L-1}, update).
 //
@@ -54,6 +55,10 @@ struct ChunkGeo {
     // corrections), u^T hi / lo, the product (k / Dc) [a o Dc ; q o Dc]^T that gives A and M
     static constexpr uint32_t kHi = 0, kLo = 128, kUpd = 256, kDW = 384, kDWc = 416, kUHi = 448,
                               kULo = 464, kAM = 480;
+    // The correction products of A and M (hi*lo + lo*hi) accumulate apart from hi*hi, in the
+    // update's columns: those are free from the state combine of one block to the update
+    // product of the next, and A and M are read out before that product is issued.
+    static constexpr uint32_t kAMc = kUpd;
     static constexpr uint32_t kCols = 512;
     // Operand tiles (K-major core matrices, see qs_tc.cuh).  A K-chunk is padded by 16 bytes
     // where a warp writes one column of consecutive key rows, so the writes spread over all
@@ -81,7 +86,6 @@ struct ChunkGeo {
     static constexpr uint32_t oStg = oBar + 32;
     static constexpr uint32_t sK = 0, sQ = L * D * 4, sS = 2 * L * D * 4, sB = 3 * L * D * 4;
     static constexpr uint32_t kBytes = oStg + sB + 3 * L * 4;
-    static constexpr int kWaitPolls = 1 << 24;
 };
 static_assert(ChunkGeo::oBwHi % 16 == 0 && ChunkGeo::oBuHi % 16 == 0 && ChunkGeo::oBar % 16 == 0 &&
               ChunkGeo::oStg % 16 == 0, "tile alignment");
@@ -94,12 +98,13 @@ __device__ __forceinline__ volatile uint32_t* chunk_abort_word(uint8_t* cb) {
     return reinterpret_cast<volatile uint32_t*>(cb + ChunkGeo::oBar + 20);
 }
 
-// Wait for phase `parity` of a product mbarrier.  Gives up after kWaitPolls polls and then
-// sets the CTA's abort word; once that word is set every later wait of the CTA gives up at
-// once, so a product that never completes costs one limit, not one per wait.
-__device__ __forceinline__ bool chunk_wait(uint64_t* bar, uint32_t parity, volatile uint32_t* abort) {
+// Wait for phase `parity` of a product mbarrier.  Gives up after `limit` polls (the call's
+// wait_polls: kDefaultWaitPolls unless a caller lowered it) and then sets the CTA's abort word;
+// once that word is set every later wait of the CTA gives up at once, so a product that never
+// completes costs one limit, not one per wait.  A limit of 0 gives up without polling.
+__device__ __forceinline__ bool chunk_wait(uint64_t* bar, uint32_t parity, volatile uint32_t* abort, int limit) {
     if (*abort != 0u) return false;
-    for (int it = 0; it < ChunkGeo::kWaitPolls; ++it) {
+    for (int it = 0; it < limit; ++it) {
         if (tc::mbar_try_wait(bar, parity)) return true;
         if ((it & 255) == 255 && *abort != 0u) return false;
     }
@@ -133,9 +138,11 @@ __device__ __forceinline__ uint32_t chunk_setup(uint8_t* cb) {
 
 // Frees the TMEM columns.  If a wait gave up (the abort word, uniform after the barrier),
 // products may still be in flight: both issuing threads commit to the teardown mbarrier and
-// warp 0 waits for it, bounded, before the columns are freed.  Copies in flight are waited
-// for too.
-__device__ __forceinline__ void chunk_teardown(uint32_t tmem, uint8_t* cb) {
+// warp 0 waits for it, bounded by the default limit whatever the call's own limit, before the
+// columns are freed.  If that wait gives up too, QS_DEV_TEARDOWN is raised: the columns are
+// freed all the same (holding them would block the next CTA's allocation for good), and the
+// host then treats the device as unusable.  Copies in flight are waited for too.
+__device__ __forceinline__ void chunk_teardown(uint32_t tmem, uint8_t* cb, int* status) {
     const int tid = threadIdx.x;
     cp_async_wait_all();
     tc::fence_before_sync();
@@ -143,7 +150,8 @@ __device__ __forceinline__ void chunk_teardown(uint32_t tmem, uint8_t* cb) {
     if (*chunk_abort_word(cb) != 0u) {
         uint64_t* bar = reinterpret_cast<uint64_t*>(cb + ChunkGeo::oBar) + 3;
         if (tid == 0 || tid == 32) tc::mma_commit(bar);
-        if (tid < 32) tc::mbar_wait(bar, 0u, ChunkGeo::kWaitPolls);
+        if (tid < 32 && !tc::mbar_wait(bar, 0u, kDefaultWaitPolls) && tid == 0)
+            raise_status(status, QS_DEV_TEARDOWN);
     }
     if (tid < 32) {
         tc::fence_after_sync();
@@ -183,7 +191,7 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
     // `phase` carries both mbarriers' parities: bit 0 the first's, bit 1 the second's
     volatile uint32_t* abort = chunk_abort_word(cb);
     auto wait_mma = [&](int which) {
-        if (!chunk_wait(bar + which, (phase >> which) & 1u, abort)) raise_status(p.status, QS_DEV_TIMEOUT);
+        if (!chunk_wait(bar + which, (phase >> which) & 1u, abort, p.wait_polls)) raise_status(p.status, QS_DEV_TIMEOUT);
         phase ^= 1u << which;
         tc::fence_after_sync();
     };
@@ -441,8 +449,8 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
                 for (int ks = 0; ks < D / 8; ++ks) {
                     const uint32_t acc = ks > 0 ? 1u : 0u;
                     tc::mma_tf32_ss(tmem + G::kAM, ah, bh, idAM, acc);
-                    tc::mma_tf32_ss(tmem + G::kAM, ah, bl, idAM, 1u);
-                    tc::mma_tf32_ss(tmem + G::kAM, al, bh, idAM, 1u);
+                    tc::mma_tf32_ss(tmem + G::kAMc, ah, bl, idAM, acc);
+                    tc::mma_tf32_ss(tmem + G::kAMc, al, bh, idAM, 1u);
                     bh += kStepW;
                     bl += kStepW;
                     ah += kStepH;
@@ -455,14 +463,16 @@ __device__ __forceinline__ void chunk_interval(const StepParams& p, Stage& S, fl
         if (!last) phase_a(t0 + L, ra);
         wait_mma(0);
         if (warp == 0) {
-            // A and M to shared memory (lane s < L holds row s of the product)
-            float x[L], y[L];
+            // A and M to shared memory (lane s < L holds row s of the product): the hi*hi
+            // accumulator plus the corrections' (one FP32 rounding)
+            float x[L], y[L], xc[L], yc[L];
             tc::tmem_ld2x16(tl + G::kAM, tl + G::kAM + L, x, y);
+            tc::tmem_ld2x16(tl + G::kAMc, tl + G::kAMc + L, xc, yc);
             if (lane < L) {
 #pragma unroll
                 for (int t = 0; t < L; ++t) {
-                    amA[t * L + lane] = x[t];
-                    amM[t * L + lane] = y[t];
+                    amA[t * L + lane] = __fadd_rn(x[t], xc[t]);
+                    amM[t * L + lane] = __fadd_rn(y[t], yc[t]);
                 }
             }
         }

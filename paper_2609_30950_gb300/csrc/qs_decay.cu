@@ -111,13 +111,14 @@ cudaError_t launch_quant_decay(const float* s, long long count, int nchan, int g
     const int L = 1 << g;
     const long long total = count * nchan;
     decay_init_kernel<<<(nchan + 255) / 256, 256, 0, stream>>>(lut, nchan, L);
-    // S = a multiple of lcm(nchan, 256) near 152 SMs x 8 x 256 threads
+    // S = a multiple of lcm(nchan, 256) near (SMs x 8) CTAs of 256 threads
     const long long lcm = static_cast<long long>(nchan) / gcd_ll(nchan, 256) * 256;
-    long long S = std::max(lcm, (311296LL / lcm) * lcm);
+    const long long target = static_cast<long long>(device_sm_count()) * 8 * 256;
+    long long S = std::max(lcm, (target / lcm) * lcm);
     while (S / 256 > 0x7fffffffLL) S -= lcm;
     decay_minmax_kernel<<<static_cast<unsigned>(S / 256), 256, 0, stream>>>(s, total, nchan, L, lut, status);
     decay_levels_kernel<<<(nchan + 127) / 128, 128, 0, stream>>>(lut, thr, nchan, L, status);
-    const unsigned blocks = 152 * 8;
+    const unsigned blocks = static_cast<unsigned>(device_sm_count()) * 8u;
     if (nchan % 4 == 0 && (reinterpret_cast<uintptr_t>(s) & 15) == 0 &&
         (reinterpret_cast<uintptr_t>(codes) & 3) == 0) {
         switch (L - 1) {
@@ -145,23 +146,29 @@ namespace {
 constexpr int kMaxDev = 64;
 std::mutex g_scratch_mu;
 float* g_scratch_addr[kMaxDev] = {};
+unsigned long long g_scratch_ctx[kMaxDev] = {};
 }  // namespace
 
 long long quant_decay_scratch_capacity() { return kDecayScratchFloats; }
 
 // Device address of the threshold scratch on the current device, looked up on the first call
-// made with that device current (a host-side lookup: make it before any stream capture).
+// made with that device current (a host-side lookup: make it before any stream capture), and
+// again whenever the device's context has been created anew since (its module, and with it
+// the array, may then sit at another address).
 cudaError_t quant_decay_scratch(float** out) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= kMaxDev) return cudaErrorInvalidDevice;
     std::lock_guard<std::mutex> lock(g_scratch_mu);
-    if (!g_scratch_addr[dev]) {
+    unsigned long long ctx = 0;
+    const bool known = current_context_id(&ctx);
+    if (!g_scratch_addr[dev] || !known || ctx != g_scratch_ctx[dev]) {
         void* ptr = nullptr;
         e = cudaGetSymbolAddress(&ptr, g_decay_thr_scratch);
         if (e != cudaSuccess) return e;
         g_scratch_addr[dev] = static_cast<float*>(ptr);
+        g_scratch_ctx[dev] = current_context_id(&ctx) ? ctx : 0ull;
     }
     *out = g_scratch_addr[dev];
     return cudaSuccess;

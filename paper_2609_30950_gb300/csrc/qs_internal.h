@@ -14,7 +14,12 @@ enum : int {
     QS_DEV_RATE = 2,    // a decay rate is not a positive finite number
     QS_DEV_TIMEOUT = 4, // a tensor-core product did not signal completion in time
     QS_DEV_CHUNK = 8,   // chunked form: a row's decay over a 16-token block leaves FP32 range
+    QS_DEV_TEARDOWN = 16,  // chunked form: after a timeout, the wait for the products still in
+                           // flight before freeing tensor memory also gave up
 };
+
+// Default limit of the chunked form's bounded mbarrier waits (polls of mbarrier.try_wait).
+constexpr int kDefaultWaitPolls = 1 << 24;
 
 constexpr int kNFit = 16;
 
@@ -34,6 +39,7 @@ struct StepParams {
     long long region_bytes;
     int stage_bytes;  // shared-memory staging capacity for one head's rows (dk dv bmax / 8)
     float alpha;      // EMA weight 2 / (span + 1)
+    int wait_polls;   // limit of the chunked form's waits for its tensor-core products (>= 0)
     // packed source / destination
     const uint8_t* in_payload;
     const uint16_t* in_scales;
@@ -91,5 +97,9 @@ cudaError_t launch_quant_decay(const float* s, long long count, int nchan, int g
                                cudaStream_t stream);
 long long quant_decay_scratch_capacity();
 cudaError_t quant_decay_scratch(float** out);
+// identity of the current CUDA context (false if unknown); see qs_api.cu
+bool current_context_id(unsigned long long* id);
+// streaming multiprocessors of the current device (cached per device)
+int device_sm_count();
 
 }  // namespace qs

@@ -82,6 +82,7 @@ struct alignas(16) WbSmem {
         float red[2][NW][DV];             // p and r partials per warp (token phase)
         float2 cand[NW][32 / (DV / 32)][kNFit + 1];   // per warp and row: (1/Delta_k, -Delta_k)
                                                       // (rows padded against bank conflicts)
+        int hist[17 * kNFit + 16];        // prep: counting sort of the rows (width, factor)
     } rc;
     float4 deqAS[DK];                     // (-A, -A, S, S) and (B, B): x = (2^23 + u - A) S + B,
     float2 deqB[DK];                      // as pairs, the operands of packed FP32 arithmetic
@@ -439,34 +440,49 @@ __global__ void __launch_bounds__(NW * 32, CHUNK ? 1 : 2) wb_row_kernel(const Wb
             const float kq = warp_sum(kk * S.q[i]);
             if (lane == 0) sm.wsum[0][(tid - 64) >> 5] = kq;
         } else if (warp == 6) {
-            // Rows in order of output width, any order within a width.  Widths 2..16 come
-            // first in ascending order (the narrowest rows have the longest range-factor
-            // search), then widths 1 and 0, so that the write-back's batches are claimed
-            // longest first.  A ballot per width present and slot gives every row its place.
-            constexpr int PER = DK / 32;
-            int key[PER], pos[PER];
-            unsigned present = 0u;
+            // Rows in order of output width, and within a width in order of the factor fitted
+            // at the previous write-back (a close predictor of this one's), any order among
+            // equals.  Widths 2..16 come first in ascending order (the narrowest rows have the
+            // longest range-factor search), then widths 1 and 0; within a width the smaller
+            // factors first (the search runs from the largest factor down, so they search
+            // longest).  The write-back claims batches of rows in this order: longest first,
+            // and the rows of a batch stop their searches at similar candidates.  A counting
+            // sort: histogram of the 17 x 16 keys, exclusive scan, ranks from the atomics.
+            constexpr int PER = DK / 32, NK = 17 * kNFit, KPL = (NK + 31) / 32;
+            int* hist = sm.rc.hist;
+            for (int k = lane; k < NK; k += 32) hist[k] = 0;
+            __syncwarp();
+            int key[PER], rank[PER];
 #pragma unroll
             for (int jj = 0; jj < PER; ++jj) {
-                key[jj] = (min(static_cast<int>(S.w_out[lane * PER + jj]), 16) + 15) % 17;
-                pos[jj] = 0;
-                present |= 1u << key[jj];
+                const int i = lane * PER + jj;
+                key[jj] = ((min(static_cast<int>(S.w_out[i]), 16) + 15) % 17) * kNFit + (S.fidx[i] & (kNFit - 1));
+                rank[jj] = atomicAdd(&hist[key[jj]], 1);
             }
-            present = __reduce_or_sync(kFull, present);
-            const unsigned lt = (1u << lane) - 1u;
-            int base = 0;
-            while (present != 0u) {
-                const int kb = __ffs(present) - 1;
-                present &= present - 1u;
+            __syncwarp();
+            int cnt[KPL], sum = 0;
 #pragma unroll
-                for (int jj = 0; jj < PER; ++jj) {
-                    const unsigned m = __ballot_sync(kFull, key[jj] == kb);
-                    if (key[jj] == kb) pos[jj] = base + __popc(m & lt);
-                    base += __popc(m);
-                }
+            for (int m = 0; m < KPL; ++m) {
+                const int k = lane * KPL + m;
+                cnt[m] = sum;
+                sum += k < NK ? hist[k] : 0;
             }
+            int incl = sum;
 #pragma unroll
-            for (int jj = 0; jj < PER; ++jj) sm.ord_out[pos[jj]] = static_cast<uint8_t>(lane * PER + jj);
+            for (int o = 1; o < 32; o <<= 1) {
+                const int n = __shfl_up_sync(kFull, incl, o);
+                if (lane >= o) incl += n;
+            }
+            __syncwarp();
+#pragma unroll
+            for (int m = 0; m < KPL; ++m) {
+                const int k = lane * KPL + m;
+                if (k < NK) hist[k] = incl - sum + cnt[m];
+            }
+            __syncwarp();
+#pragma unroll
+            for (int jj = 0; jj < PER; ++jj)
+                sm.ord_out[hist[key[jj]] + rank[jj]] = static_cast<uint8_t>(lane * PER + jj);
             if (lane == 0) sm.bat_next = NW;
         }
         __syncthreads();                                                               // B2
@@ -904,7 +920,7 @@ __global__ void __launch_bounds__(NW * 32, CHUNK ? 1 : 2) wb_row_kernel(const Wb
             }
         }
     }
-    if constexpr (CHUNK) chunk_teardown(tmem, cb);
+    if constexpr (CHUNK) chunk_teardown(tmem, cb, p.status);
 }
 
 template <int DK, int DV, int NW, bool CHUNK = false>

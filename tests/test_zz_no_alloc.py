@@ -56,6 +56,35 @@ def test_noalloc_after_a_larger_table(qs):
         assert np.array_equal(l_new.view(np.uint32), l_ref.view(np.uint32))
 
 
+def test_noalloc_at_the_largest_table_that_fits(qs):
+    # 257 heads x 255 thresholds (per-head rates, gate_bits = 8) = 65535: the largest table the
+    # configuration limits allow at or below the 65536-entry array (65536 itself would need
+    # 65536 channels at one threshold each); bit for bit against the caller-buffer entry point,
+    # twice in a row
+    for call in range(2):
+        w = synth.scaled(synth.WORKLOADS["gdn_decode"], B=2, H=257, T=5, gate_bits=8, seed=31 + call)
+        assert w.H * (2 ** w.gate_bits - 1) == 65535
+        c_ref, l_ref = _quantise(qs, w, noalloc=False)
+        c_new, l_new = _quantise(qs, w, noalloc=True)
+        assert np.array_equal(c_new, c_ref)
+        assert np.array_equal(l_new.view(np.uint32), l_ref.view(np.uint32))
+
+
+@pytest.mark.parametrize("H", [258, 1024])
+def test_noalloc_rejects_one_channel_over(qs, H):
+    # 258 heads x 255 = 65790 thresholds: one channel past the array
+    w = synth.scaled(synth.WORKLOADS["gdn_decode"], B=1, H=H, T=2, gate_bits=8)
+    cfg = qs.Config.from_workload(w)
+    s = torch.ones((1, 2, H), dtype=torch.float32, device="cuda")
+    codes = torch.full(s.shape, 7, dtype=torch.uint8, device="cuda")
+    lut = torch.zeros(H * 256, dtype=torch.float32, device="cuda")
+    with pytest.raises(qs.QstateError) as e:
+        qs.qstate_quant_decay_noalloc(cfg, s, codes, lut)
+    assert e.value.code == qs.QSTATE_EINVAL
+    qs.qstate_check()
+    assert bool((codes == 7).all()) and bool((lut == 0).all())
+
+
 def test_noalloc_rejects_tables_above_its_maximum(qs):
     # 4096 channels x (2^5 - 1) = 126976 thresholds > 65536
     w = synth.scaled(synth.WORKLOADS["kda_decode"], B=1, T=2, gate_bits=5)
