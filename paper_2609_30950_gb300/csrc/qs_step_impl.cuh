@@ -504,6 +504,12 @@ cudaError_t launch_step_shape(const qstate_cfg& cfg, int src_packed, int dst_pac
     const bool head = cfg.unit_kind == QSTATE_UNIT_HEAD && (src_packed || dst_packed);
     if (head) {   // head unit: the kernel whose lanes own whole scale groups
         if constexpr (HeadGeom<DK, DV>::ok) {
+            // a write-back whose per-head arrays are 16-byte aligned: the persistent kernel,
+            // which copies the next head's inputs with cp.async while a head computes
+            auto a16 = [](const void* q) { return q == nullptr || (reinterpret_cast<uintptr_t>(q) & 15u) == 0; };
+            if (src_packed && dst_packed && p.t_end > p.t_begin && p.in_fidx && a16(p.in_payload) &&
+                a16(p.out_payload) && a16(p.in_scales) && a16(p.in_fidx) && a16(p.k) && a16(p.q) && a16(p.v))
+                return launch_head_wb_t<DK, DV>(cfg, p, stream);
             if (src_packed && dst_packed) return launch_head_t<DK, DV, true, true>(cfg, p, stream);
             if (!src_packed && dst_packed) return launch_head_t<DK, DV, false, true>(cfg, p, stream);
             return launch_head_t<DK, DV, true, false>(cfg, p, stream);
