@@ -74,6 +74,8 @@ _CORE = ("qs_wb_row.cuh", "qs_common.cuh", "qs_internal.h")
 TRAFFIC_PROFILES = {
     ("kda_decode", "token"): ("writeback_kda_decode.md", _CORE),
     ("kda_prefill", "chunk"): ("writeback_kda_prefill_chunk.md", _CORE + ("qs_chunk.cuh", "qs_tc.cuh")),
+    ("gdn_decode", "token"): ("head_kernel_gdn_decode.md", ("qs_head.cuh", "qs_common.cuh", "qs_internal.h")),
+    ("mamba2_decode", "token"): ("writeback_mamba2_decode.md", _CORE),
 }
 
 
