@@ -319,6 +319,8 @@ def main():
                     help="tokens per host-staging chunk of the end-to-end run (default: 64 when the "
                          "state is written back every token, else max(256, C))")
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--scan-partitions", type=int, default=0,
+                    help="batch partitions of each scan, one stream each (0: the library's choice)")
     ap.add_argument("--workload", default=WORKLOAD, choices=sorted(synth.WORKLOADS),
                     help="the paper's layer shape to run (default: KDA decode)")
     args = ap.parse_args()
@@ -363,6 +365,8 @@ def main():
     st = q.new_stats(cfg, dev)
     X = q.Inputs(x["q"], x["k"], x["v"], None if coded else x["s"], codes, lut, beta, w.T)
     stream = torch.cuda.current_stream(dev)
+    q.qstate_set_scan_partitions(args.scan_partitions)
+    parts = q.qstate_scan_partition_count(cfg, X, st)
 
     def quant_decay(s):
         if coded:
@@ -467,7 +471,7 @@ def main():
 
     # decay quantiser (4), init (alloc + pack), then per write-back: write-back + alloc, or with
     # current-statistics allocation a statistics pass + alloc + write-back
-    launches_per_step = (4 if coded else 0) + 2 + (3 if args.alloc_mode == 1 else 2) * n_wb
+    launches_per_step = (4 if coded else 0) + 2 + (3 if args.alloc_mode == 1 else 2) * n_wb * parts
     clocks = clk.summary()
     if rank != 0:
         if world > 1:
@@ -494,6 +498,7 @@ def main():
         "e2e": e2e, "gpu_launches": launches_per_step * args.steps, "clocks": clocks,
         "cpu_baseline": cpu,
     }
+    line["config"]["scan_partitions"] = parts
     print(json.dumps(line))
     if world > 1:
         dist.barrier()

@@ -289,6 +289,25 @@ int qstate_check(void* stream);
  * default.  Always QSTATE_OK.  Not part of the paper's method: a diagnostic of this library. */
 int qstate_set_wait_limit(int32_t polls);
 
+/* Batch partitions of qstate_scan for the calls that follow (process-wide; read when a call is
+ * enqueued).  The batch elements of a scan are independent problems (Eq. 1 and the allocation
+ * of Sec. 3 act on each element's own state and budget), so a scan may run as n contiguous
+ * partitions of the batch, each its own chain of write-back and allocation launches on a
+ * library-owned stream, forked from the caller's stream and joined back into it by events
+ * before the call's work is complete on that stream; the chains fill each other's idle SMs.
+ * The results are bit for bit those of one chain.  n in 1..8 requests n partitions (at most
+ * one per batch element, fewer where a partition would start off a 16-byte boundary in any
+ * array); 0 (the default) chooses 4 for the token form and 2 for the chunked form.  Calls
+ * from several host threads on one device enqueue their partitioned scans one at a time.
+ * QSTATE_OK, or QSTATE_EINVAL for n outside 0..8.  Not part of the paper's method: a
+ * scheduling choice of this library. */
+int qstate_set_scan_partitions(int32_t n);
+
+/* The number of batch partitions qstate_scan would use for these arguments under the current
+ * request (1 = one chain on the caller's stream), or 0 if cfg, x or stats is invalid.  No
+ * launch. */
+int qstate_scan_partition_count(const qstate_cfg* cfg, const qstate_inputs* x, const qstate_stats* stats);
+
 /* Message for the last failure on this host thread ("" if none).  Valid until the next call. */
 const char* qstate_last_error(void);
 

@@ -60,7 +60,8 @@ EXPORTS = ["qstate_validate", "qstate_region_bytes", "qstate_units", "qstate_sca
            "qstate_bits_per_element", "qstate_init", "qstate_alloc_bits", "qstate_pack",
            "qstate_unpack", "qstate_quant_decay", "qstate_quant_decay_noalloc", "qstate_step",
            "qstate_scan", "qstate_scan_host",
-           "qstate_scan_fp32", "qstate_check", "qstate_set_wait_limit", "qstate_last_error"]
+           "qstate_scan_fp32", "qstate_check", "qstate_set_wait_limit", "qstate_set_scan_partitions",
+           "qstate_scan_partition_count", "qstate_last_error"]
 
 _lib = None
 
@@ -107,6 +108,8 @@ def load(path: str | None = None, build_if_missing: bool = False):
     L.qstate_scan_fp32.argtypes = [PC, P, ct.POINTER(_Inputs), ct.c_int32, ct.c_int32, P, P]
     L.qstate_check.argtypes = [P]
     L.qstate_set_wait_limit.argtypes = [ct.c_int32]
+    L.qstate_set_scan_partitions.argtypes = [ct.c_int32]
+    L.qstate_scan_partition_count.argtypes = [ct.c_void_p, ct.c_void_p, ct.c_void_p]
     L.qstate_last_error.restype = ct.c_char_p
     for name in EXPORTS:
         if name not in ("qstate_region_bytes", "qstate_units", "qstate_scale_groups",
@@ -360,3 +363,15 @@ def qstate_set_wait_limit(polls: int) -> None:
     """Limit of the chunked form's waits for its tensor-core products in later calls (polls;
     0 gives up at once, negative restores the default)."""
     _check(_lib_or_raise().qstate_set_wait_limit(int(polls)))
+
+
+def qstate_set_scan_partitions(n: int) -> None:
+    """Batch partitions of later scans, each on its own stream (1..8; 0 chooses per
+    configuration).  Results are identical for every choice."""
+    _check(_lib_or_raise().qstate_set_scan_partitions(int(n)))
+
+
+def qstate_scan_partition_count(cfg: Config, x: Inputs, stats: Stats) -> int:
+    """Batch partitions a scan with these arguments would use now (0 if they are invalid)."""
+    c, xi, st = cfg.c(), x.c(), stats.c()
+    return int(_lib_or_raise().qstate_scan_partition_count(ct.byref(c), ct.byref(xi), ct.byref(st)))

@@ -331,6 +331,137 @@ int run_alloc(const qstate_cfg* c, const float* ms, const float* mr, const float
     return e == cudaSuccess ? QSTATE_OK : cuda_fail(e, "allocation kernel");
 }
 
+// ---- a scan as concurrent batch partitions ------------------------------------------------------
+// The batch elements of a scan are independent problems: Eq. (1), the statistics and the
+// allocation of Sec. 3 act on each element's own state and budget.  qstate_scan may therefore
+// run G contiguous batch partitions, each a chain of write-back and allocation launches on a
+// stream of its own, forked from the caller's stream and joined back into it by events.  The
+// chains fill each other's idle SMs (the last wave of a launch, and the allocation launches,
+// which occupy one CTA per batch element).  Every kernel computes each head and batch element on
+// its own, so the results are those of one chain bit for bit.
+constexpr int kMaxParts = 8;
+struct PartStreams {
+    bool ready = false;
+    unsigned long long ctx = 0;
+    cudaStream_t s[kMaxParts] = {};          // s[0] unused: partition 0 runs on the caller's stream
+    cudaEvent_t fork = nullptr;
+    cudaEvent_t join[kMaxParts] = {};
+};
+PartStreams g_parts[kMaxDevices];
+// The fork and join events are shared by the calls on a device: a partitioned scan is enqueued
+// under this lock (the enqueue only, not the work).
+std::mutex g_part_mu;
+// Partitions requested by qstate_set_scan_partitions (0: chosen per configuration).
+std::atomic<int> g_scan_parts{0};
+
+// Streams and events of the current device, created once per device and context.  Caller holds
+// g_part_mu.
+int part_streams(PartStreams** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= kMaxDevices) return fail(QSTATE_EDEVICE, "device index %d out of range", dev);
+    unsigned long long ctx = 0;
+    const bool known = current_context_id(&ctx);
+    PartStreams& P = g_parts[dev];
+    if (!P.ready || !known || ctx != P.ctx) {
+        // handles of an earlier context went with it; nothing to destroy
+        P = PartStreams{};
+        for (int i = 1; i < kMaxParts; ++i)
+            if ((e = cudaStreamCreateWithFlags(&P.s[i], cudaStreamNonBlocking)) != cudaSuccess)
+                return cuda_fail(e, "partition stream");
+        if ((e = cudaEventCreateWithFlags(&P.fork, cudaEventDisableTiming)) != cudaSuccess)
+            return cuda_fail(e, "partition event");
+        for (int i = 1; i < kMaxParts; ++i)
+            if ((e = cudaEventCreateWithFlags(&P.join[i], cudaEventDisableTiming)) != cudaSuccess)
+                return cuda_fail(e, "partition event");
+        P.ctx = known ? ctx : 0ull;
+        P.ready = known;   // an unknown context is asked again next time
+    }
+    *out = &P;
+    return QSTATE_OK;
+}
+
+// Bytes per batch element of every array a scan touches, with the partition's view of them.
+struct ScanArrays {
+    qstate_buf ping, pong;
+    qstate_inputs x;
+    float* o;
+    qstate_stats st;
+};
+
+long long elem_offset_low_bits(const qstate_cfg* c, const qstate_inputs* x, const qstate_stats* st,
+                                      long long b0) {
+    // OR of the byte offsets of batch element b0 in every array: 16-byte aligned iff its low
+    // four bits are zero
+    const long long T = x->T, H = c->H, dk = c->dk, dv = c->dv;
+    const long long units = units_of(c), groups = groups_of(c);
+    const long long ns = c->decay_kind == QSTATE_DECAY_ROW ? T * H * dk : T * H;
+    long long m = b0 * region_of(c);
+    m |= b0 * groups * 2;
+    m |= b0 * units;
+    m |= b0 * H * 4;
+    m |= b0 * groups;
+    if (st) m |= b0 * units * 4;
+    m |= b0 * T * H * dk * 4;
+    m |= b0 * T * H * dv * 4;
+    m |= x->s_code ? b0 * ns : b0 * ns * 4;
+    if (x->beta) m |= b0 * T * H * 4;
+    return m & 15;
+}
+
+ScanArrays slice(const qstate_cfg* c, const qstate_buf* ping, const qstate_buf* pong, const qstate_inputs* x,
+                 float* o, const qstate_stats* st, long long b0) {
+    const long long T = x->T, H = c->H, dk = c->dk, dv = c->dv;
+    const long long units = units_of(c), groups = groups_of(c), region = region_of(c);
+    const long long ns = c->decay_kind == QSTATE_DECAY_ROW ? T * H * dk : T * H;
+    auto buf = [&](const qstate_buf* b) {
+        qstate_buf r;
+        r.payload = b->payload + b0 * region;
+        r.scales = b->scales + b0 * groups;
+        r.widths = b->widths + b0 * units;
+        r.head_off = b->head_off + b0 * H;
+        r.fidx = b->fidx + b0 * groups;
+        return r;
+    };
+    ScanArrays a;
+    a.ping = buf(ping);
+    a.pong = buf(pong);
+    a.x = *x;
+    a.x.q = x->q + b0 * T * H * dk;
+    a.x.k = x->k + b0 * T * H * dk;
+    a.x.v = x->v + b0 * T * H * dv;
+    if (x->s) a.x.s = x->s + b0 * ns;
+    if (x->s_code) a.x.s_code = x->s_code + b0 * ns;
+    if (x->beta) a.x.beta = x->beta + b0 * T * H;
+    if (x->a) a.x.a = x->a + b0 * T * H * dk;
+    if (x->w) a.x.w = x->w + b0 * T * H * dv;
+    a.o = o + b0 * T * H * dv;
+    a.st.ema_s = st->ema_s + b0 * units;
+    a.st.ema_r = st->ema_r + b0 * units;
+    a.st.range = st->range ? st->range + b0 * units : nullptr;
+    return a;
+}
+
+// Partitions of a scan: the requested number, else the count measured best on GB300 for the
+// benchmark layer shapes (token form 4: 6 % per token at KDA decode, 24 % at Gated DeltaNet;
+// chunked form 2: 10 % at KDA prefill, where 3 or 4 split its 16 batch elements less evenly over
+// the one-CTA-per-SM launches); at most one per batch element, and fewer where a partition would
+// start off a 16-byte boundary in any array.
+int scan_parts(const qstate_cfg* c, const qstate_inputs* x, const qstate_stats* st) {
+    int G = g_scan_parts.load();
+    if (G <= 0) G = c->interval_form == QSTATE_FORM_CHUNK ? 2 : 4;
+    G = G < kMaxParts ? G : kMaxParts;
+    G = G < c->B ? G : c->B;
+    for (; G > 1; --G) {
+        bool ok = true;
+        for (int p = 1; p < G && ok; ++p)
+            ok = elem_offset_low_bits(c, x, st, static_cast<long long>(c->B) * p / G) == 0;
+        if (ok) break;
+    }
+    return G;
+}
+
 }  // namespace
 
 extern "C" {
@@ -538,20 +669,77 @@ int qstate_scan(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong, const
     int rc = validate(cfg);
     if (rc) return rc;
     if ((rc = check_inputs(cfg, x, t_begin, t_end, o))) return rc;
-    qstate_buf* src = ping;
-    qstate_buf* dst = pong;
-    int in_pong = 0;
-    int w = w_index0;
-    for (int t0 = t_begin; t0 < t_end; t0 += cfg->C) {
-        const int t1 = t0 + cfg->C < t_end ? t0 + cfg->C : t_end;
-        rc = qstate_step(cfg, src, dst, x, t0, t1, w++, o, stats, stream);
-        if (rc) return rc;
-        qstate_buf* tmp = src;
-        src = dst;
-        dst = tmp;
-        in_pong ^= 1;
+    if (!buf_ok(ping) || !buf_ok(pong)) return fail(QSTATE_EINVAL, "null buffer pointer");
+    if (!stats || !stats->ema_s || !stats->ema_r || (cfg->unit_kind == QSTATE_UNIT_ROW && !stats->range))
+        return fail(QSTATE_EINVAL, "null statistics pointer");
+    const int nsteps = t_end > t_begin ? (t_end - t_begin + cfg->C - 1) / cfg->C : 0;
+    const int G = nsteps > 0 ? scan_parts(cfg, x, stats) : 1;
+    if (G <= 1) {
+        qstate_buf* src = ping;
+        qstate_buf* dst = pong;
+        int w = w_index0;
+        for (int t0 = t_begin; t0 < t_end; t0 += cfg->C) {
+            const int t1 = t0 + cfg->C < t_end ? t0 + cfg->C : t_end;
+            rc = qstate_step(cfg, src, dst, x, t0, t1, w++, o, stats, stream);
+            if (rc) return rc;
+            qstate_buf* tmp = src;
+            src = dst;
+            dst = tmp;
+        }
+        if (final_in_pong) *final_in_pong = nsteps & 1;
+        return QSTATE_OK;
     }
-    if (final_in_pong) *final_in_pong = in_pong;
+    // batch partitions [B p / G, B (p + 1) / G), one stream each (partition 0 on the caller's)
+    int* status = nullptr;
+    if ((rc = acquire_status(&status))) return rc;   // also makes the context current
+    std::lock_guard<std::mutex> lock(g_part_mu);
+    PartStreams* P = nullptr;
+    if ((rc = part_streams(&P))) return rc;
+    cudaStream_t cs = static_cast<cudaStream_t>(stream);
+    qstate_cfg sub[kMaxParts];
+    ScanArrays arr[kMaxParts];
+    cudaStream_t ps[kMaxParts];
+    for (int p = 0; p < G; ++p) {
+        const long long b0 = static_cast<long long>(cfg->B) * p / G, b1 = static_cast<long long>(cfg->B) * (p + 1) / G;
+        sub[p] = *cfg;
+        sub[p].B = static_cast<int32_t>(b1 - b0);
+        arr[p] = slice(cfg, ping, pong, x, o, stats, b0);
+        ps[p] = p == 0 ? cs : P->s[p];
+    }
+    cudaError_t e = cudaEventRecord(P->fork, cs);
+    for (int p = 1; p < G && e == cudaSuccess; ++p) e = cudaStreamWaitEvent(ps[p], P->fork, 0);
+    if (e != cudaSuccess) return cuda_fail(e, "partition fork");
+    int w = w_index0, flip = 0;
+    for (int t0 = t_begin; t0 < t_end && rc == QSTATE_OK; t0 += cfg->C, ++w, flip ^= 1) {
+        const int t1 = t0 + cfg->C < t_end ? t0 + cfg->C : t_end;
+        for (int p = 0; p < G && rc == QSTATE_OK; ++p) {
+            qstate_buf* src = flip ? &arr[p].pong : &arr[p].ping;
+            qstate_buf* dst = flip ? &arr[p].ping : &arr[p].pong;
+            rc = qstate_step(&sub[p], src, dst, &arr[p].x, t0, t1, w, arr[p].o, &arr[p].st, ps[p]);
+        }
+    }
+    // join, also after a failed step, so that no partition's work is left unordered
+    e = cudaSuccess;
+    for (int p = 1; p < G; ++p) {
+        cudaError_t e1 = cudaEventRecord(P->join[p], ps[p]);
+        if (e1 == cudaSuccess) e1 = cudaStreamWaitEvent(cs, P->join[p], 0);
+        if (e == cudaSuccess) e = e1;
+    }
+    if (rc) return rc;
+    if (e != cudaSuccess) return cuda_fail(e, "partition join");
+    if (final_in_pong) *final_in_pong = nsteps & 1;
+    return QSTATE_OK;
+}
+
+int qstate_scan_partition_count(const qstate_cfg* cfg, const qstate_inputs* x, const qstate_stats* stats) {
+    if (validate(cfg) != QSTATE_OK || !x || !x->q || !x->k || !x->v || !stats || !stats->ema_s || !stats->ema_r)
+        return 0;
+    return scan_parts(cfg, x, stats);
+}
+
+int qstate_set_scan_partitions(int32_t n) {
+    if (n < 0 || n > kMaxParts) return fail(QSTATE_EINVAL, "partitions must be in [0, %d]", kMaxParts);
+    g_scan_parts.store(n);
     return QSTATE_OK;
 }
 

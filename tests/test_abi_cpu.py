@@ -88,3 +88,12 @@ def test_chunked_form_configuration_limits(lib):
         with pytest.raises(q.QstateError) as e:
             q.validate(q.Config(**base))
         assert e.value.code == q.QSTATE_EINVAL
+
+
+def test_scan_partition_setter_checks_its_range(lib):
+    # no launch: the setter only records the request
+    from paper_2609_30950_gb300 import QSTATE_EINVAL, QSTATE_OK
+    assert lib.qstate_set_scan_partitions(9) == QSTATE_EINVAL
+    assert lib.qstate_set_scan_partitions(-1) == QSTATE_EINVAL
+    for n in (8, 1, 0):
+        assert lib.qstate_set_scan_partitions(n) == QSTATE_OK
