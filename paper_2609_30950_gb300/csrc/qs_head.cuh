@@ -71,6 +71,8 @@ __device__ __forceinline__ float hv_get(float2 v, int c) { return c == 0 ? v.x :
 __device__ __forceinline__ float hv_get(float v, int) { return v; }
 __device__ __forceinline__ void hv_set(float2& v, int c, float s) { if (c == 0) v.x = s; else v.y = s; }
 __device__ __forceinline__ void hv_set(float& v, int, float s) { v = s; }
+__device__ __forceinline__ float2 hv_abs(float2 v) { return make_float2(fabsf(v.x), fabsf(v.y)); }
+__device__ __forceinline__ float hv_abs(float v) { return fabsf(v); }
 
 template <int DK, int DV, bool SRC_PACKED, bool DST_PACKED>
 __global__ void __launch_bounds__(HeadGeom<DK, DV>::NT, 2) head_kernel(const StepParams p) {
@@ -467,6 +469,44 @@ cudaError_t launch_head_t(const qstate_cfg& cfg, const StepParams& p, cudaStream
 
 namespace qs {
 
+// Codes and packing of a head's rows (Sec. 3, "Levels and storage") at a compile-time width W
+// (one width per head, so the kernel switches once per head): the lane's CPL codes of row r
+// (offset binary for W >= 2; for W = 1 the sign bit, 1 for x < 0, negative zero counting as
+// positive) are OR-ed into the row's bit stream at bit col0 W.  A lane's CPL W bits stay within
+// one word when CPL W divides 32; at CPL W = 32 the word is the lane's alone.
+template <int W, int DV, int CPL, class V>
+__device__ __forceinline__ void head_pack_rows(const V (&x)[32], V inv2, uint8_t* pout, int r0, int col0) {
+    constexpr int rowbytes = W * (DV / 8);
+    constexpr int n = W >= 2 ? (1 << (W - 1)) - 1 : 0;
+    const int P = col0 * W, idx = P >> 5, sh = P & 31;
+    uint32_t* words = reinterpret_cast<uint32_t*>(pout + r0 * rowbytes) + idx;
+#pragma unroll
+    for (int r = 0; r < 32; ++r) {
+        uint32_t chunk = 0u;
+        if constexpr (W >= 2) {
+            const V tq = hv_add(hv_mul(x[r], inv2), hv_bc<V>(kMagic));
+#pragma unroll
+            for (int c = 0; c < CPL; ++c)
+                chunk |= static_cast<uint32_t>(__viaddmin_s32_relu(__float_as_int(hv_get(tq, c)),
+                                                                   n - static_cast<int>(kMagicBits), 2 * n)) << (c * W);
+        } else {
+#pragma unroll
+            for (int c = 0; c < CPL; ++c) chunk |= (hv_get(x[r], c) < 0.0f ? 1u : 0u) << c;
+        }
+        uint32_t* wd = reinterpret_cast<uint32_t*>(reinterpret_cast<uint8_t*>(words) + r * rowbytes);
+        if constexpr (CPL * W == 32) {
+            *wd = chunk;
+        } else if constexpr (32 % (CPL * W) == 0) {
+            if (chunk) atomicOr(wd, chunk << sh);
+        } else {
+            const uint64_t sh64 = static_cast<uint64_t>(chunk) << sh;
+            const uint32_t lo = static_cast<uint32_t>(sh64), hi = static_cast<uint32_t>(sh64 >> 32);
+            if (lo) atomicOr(wd, lo);
+            if (hi) atomicOr(wd + 1, hi);
+        }
+    }
+}
+
 // ---- persistent write-back of the head unit ---------------------------------------------------
 // The write-back kernel above (one CTA per head) loads a head's payload, steps and inputs only
 // when the CTA starts, so every head begins with a wait on global memory.  This variant keeps
@@ -800,17 +840,12 @@ __global__ void __launch_bounds__(HeadGeom<DK, DV>::NT, 2) head_wb_kernel(const 
         {
             const int w = w_out;
             const bool refit = (p.fit_every <= 1) || ((p.w_index + h) % p.fit_every == 0);
-            uint32_t sg[CPL];
             V Rg = hv_bc<V>(0.0f), Mg = hv_bc<V>(0.0f);
-#pragma unroll
-            for (int c = 0; c < CPL; ++c) sg[c] = 0u;
 #pragma unroll
             for (int r = 0; r < 32; ++r) {
 #pragma unroll
                 for (int c = 0; c < CPL; ++c) {
-                    const float xv = hv_get(x[r], c), av = fabsf(xv);
-                    sg[c] |= (xv < 0.0f ? 1u : 0u) << r;
-                    hv_set(x[r], c, av);
+                    const float av = fabsf(hv_get(x[r], c));
                     hv_set(Rg, c, fmaxf(hv_get(Rg, c), av));
                     if (w == 1) hv_set(Mg, c, __fadd_rn(hv_get(Mg, c), av));   // in row order
                 }
@@ -862,14 +897,14 @@ __global__ void __launch_bounds__(HeadGeom<DK, DV>::NT, 2) head_wb_kernel(const 
                     V a0 = hv_bc<V>(0.0f), a1 = hv_bc<V>(0.0f);
 #pragma unroll
                     for (int r = 0; r < 32; r += 2) {
-                        V t0 = hv_fma(x[r], iv, M2), t1 = hv_fma(x[r + 1], iv, M2);
+                        V t0 = hv_fma(hv_abs(x[r]), iv, M2), t1 = hv_fma(hv_abs(x[r + 1]), iv, M2);
 #pragma unroll
                         for (int c = 0; c < CPL; ++c) {
                             hv_set(t0, c, fminf(hv_get(t0, c), lim));
                             hv_set(t1, c, fminf(hv_get(t1, c), lim));
                         }
-                        const V e0 = hv_fma(hv_add(t0, nM2), nd, x[r]);
-                        const V e1 = hv_fma(hv_add(t1, nM2), nd, x[r + 1]);
+                        const V e0 = hv_fma(hv_add(t0, nM2), nd, hv_abs(x[r]));
+                        const V e1 = hv_fma(hv_add(t1, nM2), nd, hv_abs(x[r + 1]));
                         a0 = hv_fma(e0, e0, a0);
                         a1 = hv_fma(e1, e1, a1);
                     }
@@ -899,33 +934,12 @@ __global__ void __launch_bounds__(HeadGeom<DK, DV>::NT, 2) head_wb_kernel(const 
                 V inv2;
 #pragma unroll
                 for (int c = 0; c < CPL; ++c) hv_set(inv2, c, step_rcp(D[c]));
-                const int n = w >= 2 ? (1 << (w - 1)) - 1 : 0;
-                const int rowbytes = w * (DV / 8);
-                const int P = col0 * w, idx = P >> 5, sh = P & 31;
-                uint32_t* words = reinterpret_cast<uint32_t*>(pout + r0 * rowbytes) + idx;
-#pragma unroll
-                for (int r = 0; r < 32; ++r) {
-                    uint32_t chunk = 0u;
-                    if (w >= 2) {
-                        V xs;
-#pragma unroll
-                        for (int c = 0; c < CPL; ++c)
-                            hv_set(xs, c, __uint_as_float(__float_as_uint(hv_get(x[r], c)) | (((sg[c] >> r) & 1u) << 31)));
-                        const V tq = hv_add(hv_mul(xs, inv2), hv_bc<V>(kMagic));
-#pragma unroll
-                        for (int c = 0; c < CPL; ++c)
-                            chunk |= static_cast<uint32_t>(__viaddmin_s32_relu(__float_as_int(hv_get(tq, c)),
-                                                                               n - static_cast<int>(kMagicBits), 2 * n))
-                                     << (c * w);
-                    } else {
-#pragma unroll
-                        for (int c = 0; c < CPL; ++c) chunk |= ((sg[c] >> r) & 1u) << c;
-                    }
-                    uint32_t* wd = reinterpret_cast<uint32_t*>(reinterpret_cast<uint8_t*>(words) + r * rowbytes);
-                    const uint64_t sh64 = static_cast<uint64_t>(chunk) << sh;
-                    const uint32_t lo = static_cast<uint32_t>(sh64), hi = static_cast<uint32_t>(sh64 >> 32);
-                    if (lo) atomicOr(wd, lo);
-                    if (hi) atomicOr(wd + 1, hi);
+                switch (w) {
+#define QS_HP(N) case N: head_pack_rows<N, DV, CPL, V>(x, inv2, pout, r0, col0); break;
+                    QS_HP(1) QS_HP(2) QS_HP(3) QS_HP(4) QS_HP(5) QS_HP(6) QS_HP(7) QS_HP(8)
+                    QS_HP(9) QS_HP(10) QS_HP(11) QS_HP(12) QS_HP(13) QS_HP(14) QS_HP(15) QS_HP(16)
+#undef QS_HP
+                    default: break;
                 }
             }
             const size_t gb = static_cast<size_t>(bh) * NSG + soff;
