@@ -469,6 +469,35 @@ cudaError_t launch_head_t(const qstate_cfg& cfg, const StepParams& p, cudaStream
 
 namespace qs {
 
+// Decoding and dequantisation of a head's rows at a compile-time width W (the persistent
+// kernel switches once per head): the lane's CPL codes of row r sit at bit col0 W of the row, in
+// one word when CPL W divides 32, else across two; x = (2^23 + u - A) S + B as in the kernel
+// above.
+template <int W, int DV, int CPL, class V>
+__device__ __forceinline__ void head_unpack_rows(const uint8_t* pay, int r0, int col0, V A2, V S2, V B2,
+                                                 V (&x)[32]) {
+    if constexpr (W == 0) {
+#pragma unroll
+        for (int r = 0; r < 32; ++r) x[r] = hv_bc<V>(0.0f);
+    } else {
+        constexpr int rowbytes = W * (DV / 8);
+        constexpr uint32_t mask = (1u << W) - 1u;
+        const int P = col0 * W, idx = P >> 5, sh = P & 31;
+        const uint8_t* base = pay + r0 * rowbytes + 4 * idx;
+#pragma unroll
+        for (int r = 0; r < 32; ++r) {
+            const uint32_t* wd = reinterpret_cast<const uint32_t*>(base + r * rowbytes);
+            uint32_t chunk;
+            if constexpr (32 % (CPL * W) == 0) chunk = wd[0] >> sh;
+            else chunk = __funnelshift_r(wd[0], wd[1], sh);
+            V t;
+#pragma unroll
+            for (int c = 0; c < CPL; ++c) hv_set(t, c, __uint_as_float(kTwo23Bits | ((chunk >> (c * W)) & mask)));
+            x[r] = hv_fma(hv_add(t, A2), S2, B2);
+        }
+    }
+}
+
 // Codes and packing of a head's rows (Sec. 3, "Levels and storage") at a compile-time width W
 // (one width per head, so the kernel switches once per head): the lane's CPL codes of row r
 // (offset binary for W >= 2; for W = 1 the sign bit, 1 for x < 0, negative zero counting as
@@ -701,18 +730,14 @@ __global__ void __launch_bounds__(HeadGeom<DK, DV>::NT, 2) head_wb_kernel(const 
                 hv_set(B2, c, w_in == 1 ? D : 0.0f);
             }
             const V A2 = hv_bc<V>(nA);
-            const int rowbytes = w_in * (DV / 8);
-            const int P = col0 * w_in, idx = P >> 5, sh = P & 31;
-            const uint32_t mask = (1u << w_in) - 1u;
-            const uint8_t* base = pay + r0 * rowbytes + 4 * idx;
+            switch (w_in) {   // widths above 16 were rejected with the head's layout
+#define QS_HU(N) case N: head_unpack_rows<N, DV, CPL, V>(pay, r0, col0, A2, S2, B2, x); break;
+                QS_HU(0) QS_HU(1) QS_HU(2) QS_HU(3) QS_HU(4) QS_HU(5) QS_HU(6) QS_HU(7) QS_HU(8)
+                QS_HU(9) QS_HU(10) QS_HU(11) QS_HU(12) QS_HU(13) QS_HU(14) QS_HU(15) QS_HU(16)
+#undef QS_HU
+                default:
 #pragma unroll
-            for (int r = 0; r < 32; ++r) {
-                const uint32_t* wd = reinterpret_cast<const uint32_t*>(base + r * rowbytes);
-                const uint32_t chunk = w_in == 0 ? 0u : __funnelshift_r(wd[0], wd[1], sh);
-                V t;
-#pragma unroll
-                for (int c = 0; c < CPL; ++c) hv_set(t, c, __uint_as_float(kTwo23Bits | ((chunk >> (c * w_in)) & mask)));
-                x[r] = hv_fma(hv_add(t, A2), S2, B2);
+                    for (int r = 0; r < 32; ++r) x[r] = hv_bc<V>(0.0f);
             }
         }
 
