@@ -68,17 +68,22 @@ __device__ int block_exclusive_scan(int v, int* red, int* total) {
 
 }  // namespace
 
+// Group of unit u: a shift when the group size gsz is a power of two (gshift >= 0), else a
+// division.
+__device__ __forceinline__ int group_of(int u, int gsz, int gshift) { return gshift >= 0 ? u >> gshift : u / gsz; }
+
 // Allocation weight c_u (Eq. 3 and the alternatives of Table 1), one IEEE rounding per
 // operation.  ms_s / mr_s: the batch element's EMA statistics; Rs / gmean: its ranges, stored
 // with one padding word after every group of gsz units, and the group means of R^2 (row unit).
 __device__ float weight(const AllocParams& p, int u, const float* ms_s, const float* mr_s, const float* Rs,
-                        const float* gmean, int gsz) {
+                        const float* gmean, int gsz, int gshift) {
     const int kind = p.weight_kind;
     float R2 = 1.0f, rt2 = 1.0f;   // R^2 and Rtilde^2 (1 for the head unit)
     if (p.unit_row) {
-        const float R = Rs[u + u / gsz];
+        const int gi = group_of(u, gsz, gshift);
+        const float R = Rs[u + gi];
         R2 = __fmul_rn(R, R);
-        const float m = gmean[u / gsz];
+        const float m = gmean[gi];
         if (m > 0.0f) rt2 = __fdiv_rn(R2, m);
     }
     if (kind == QSTATE_WEIGHT_RANGE) return R2;
@@ -148,6 +153,7 @@ __global__ void __launch_bounds__(kThreads, 2) alloc_kernel(const AllocParams p)
     const int N = p.units;
     int* key = reinterpret_cast<int*>(smem);
     const int gsz = p.group_heads * p.dk;
+    const int gshift = (gsz & (gsz - 1)) == 0 ? __ffs(gsz) - 1 : -1;
     const int ngroups = p.unit_row ? N / gsz : 0;
     float* ms_s = reinterpret_cast<float*>(key + N);                 // EMA statistics
     float* mr_s = ms_s + N;
@@ -169,15 +175,30 @@ __global__ void __launch_bounds__(kThreads, 2) alloc_kernel(const AllocParams p)
         for (int u = tid; u < N; u += kThreads) {
             ms_s[u] = p.ema_s[base + u];
             mr_s[u] = p.ema_r[base + u];
-            if (p.unit_row) Rs[u + u / gsz] = p.range[base + u];
+            if (p.unit_row) Rs[u + group_of(u, gsz, gshift)] = p.range[base + u];
         }
         __syncthreads();
         if (p.unit_row) {
+            // one thread per group, its sum a chain of gsz dependent additions: the next 16
+            // ranges are loaded while the current 16 are added
             for (int g = tid; g < ngroups; g += kThreads) {
                 const float* rg = Rs + g * (gsz + 1);
                 float acc = 0.0f;
-#pragma unroll 8
-                for (int r = 0; r < gsz; ++r) acc = __fadd_rn(acc, __fmul_rn(rg[r], rg[r]));
+                constexpr int PF = 16;
+                float cur[PF];
+                const int full = gsz - gsz % PF;
+#pragma unroll
+                for (int k = 0; k < PF; ++k) cur[k] = k < gsz ? rg[k] : 0.0f;
+                for (int r = 0; r < full; r += PF) {
+                    float nxt[PF];
+#pragma unroll
+                    for (int k = 0; k < PF; ++k) nxt[k] = r + PF + k < gsz ? rg[r + PF + k] : 0.0f;
+#pragma unroll
+                    for (int k = 0; k < PF; ++k) acc = __fadd_rn(acc, __fmul_rn(cur[k], cur[k]));
+#pragma unroll
+                    for (int k = 0; k < PF; ++k) cur[k] = nxt[k];
+                }
+                for (int r = full; r < gsz; ++r) acc = __fadd_rn(acc, __fmul_rn(rg[r], rg[r]));
                 gmean[g] = __fdiv_rn(acc, static_cast<float>(gsz));
             }
         }
@@ -192,7 +213,7 @@ __global__ void __launch_bounds__(kThreads, 2) alloc_kernel(const AllocParams p)
     const long long M = p.total - static_cast<long long>(N) * p.bmin;
     for (int u = tid; u < N; u += kThreads) {
         float c = 1.0f;
-        if (!p.uniform) c = weight(p, u, ms_s, mr_s, Rs, gmean, gsz);
+        if (!p.uniform) c = weight(p, u, ms_s, mr_s, Rs, gmean, gsz, gshift);
         if (c > 0x1p60f) c = 0x1p60f;
         const int k = (c >= 0x1p-60f) ? __float_as_int(c) : kNullKey;
         key[u] = k;
