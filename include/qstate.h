@@ -255,8 +255,9 @@ int qstate_scan(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong,
  * chunk by token chunk, into x_dev's buffer (one copy per tensor, chunk and batch element) on
  * copy_stream, while the compute stream runs the scan of the previous chunk; inputs absent
  * from x_host (e.g. rate codes made on the device by qstate_quant_decay) must already be in
- * x_dev.  Readouts of each chunk are copied from o_dev to o_host on copy_stream once the chunk
- * is done.  chunk (tokens) is a multiple of C.  stream and copy_stream are distinct non-NULL
+ * x_dev.  Readouts of each chunk are copied from o_dev to o_host once the chunk is done, on a
+ * stream the library owns (so that they move while later chunks' inputs come in).  chunk
+ * (tokens) is a multiple of C.  stream and copy_stream are distinct non-NULL
  * streams; work on stream completes only after the last readout has reached o_host.  Host
  * memory should be pinned (pageable memory works but the copies then serialise).  Results are
  * those of qstate_scan(ping, pong, x_dev, ...) bit for bit. */

@@ -344,6 +344,7 @@ struct PartStreams {
     bool ready = false;
     unsigned long long ctx = 0;
     cudaStream_t s[kMaxParts] = {};          // s[0] unused: partition 0 runs on the caller's stream
+    cudaStream_t rd = nullptr;               // qstate_scan_host's readout copies
     cudaEvent_t fork = nullptr;
     cudaEvent_t join[kMaxParts] = {};
 };
@@ -370,6 +371,8 @@ int part_streams(PartStreams** out) {
         for (int i = 1; i < kMaxParts; ++i)
             if ((e = cudaStreamCreateWithFlags(&P.s[i], cudaStreamNonBlocking)) != cudaSuccess)
                 return cuda_fail(e, "partition stream");
+        if ((e = cudaStreamCreateWithFlags(&P.rd, cudaStreamNonBlocking)) != cudaSuccess)
+            return cuda_fail(e, "readout stream");
         if ((e = cudaEventCreateWithFlags(&P.fork, cudaEventDisableTiming)) != cudaSuccess)
             return cuda_fail(e, "partition event");
         for (int i = 1; i < kMaxParts; ++i)
@@ -763,6 +766,17 @@ int qstate_scan_host(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong,
                      (x_host->w && !x_dev->w);
     if (bad) return fail(QSTATE_EINVAL, "a host input has no device buffer");
     cudaStream_t cs = static_cast<cudaStream_t>(stream), ts = static_cast<cudaStream_t>(copy_stream);
+    // readouts go back on a library-owned stream, so that they move while later chunks'
+    // inputs come in (the host link carries both directions at once)
+    cudaStream_t rs = nullptr;
+    {
+        int* status = nullptr;
+        if ((rc = acquire_status(&status))) return rc;   // also makes the context current
+        std::lock_guard<std::mutex> lock(g_part_mu);
+        PartStreams* P = nullptr;
+        if ((rc = part_streams(&P))) return rc;
+        rs = P->rd;
+    }
     const int B = cfg->B, T = x_dev->T, H = cfg->H;
     const size_t f4 = sizeof(float);
     const size_t nchan = cfg->decay_kind == QSTATE_DECAY_ROW ? static_cast<size_t>(H) * cfg->dk : H;
@@ -774,15 +788,16 @@ int qstate_scan_host(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong,
     // tokens [t0, t1) of a (B, T, per) token-major tensor: one copy per batch element (one
     // copy in all when the chunk spans every token); plain copies move pinned host memory at
     // full link speed where strided 2D copies were measured several times slower
-    auto copy_tokens = [&](void* dst, const void* src, size_t per, int t0, int t1, cudaMemcpyKind kind) {
+    auto copy_tokens = [&](void* dst, const void* src, size_t per, int t0, int t1, cudaMemcpyKind kind,
+                           cudaStream_t cst) {
         const size_t pitch = static_cast<size_t>(T) * per, off = static_cast<size_t>(t0) * per;
         const size_t width = static_cast<size_t>(t1 - t0) * per;
         if (width == pitch)
-            return cudaMemcpyAsync(dst, src, pitch * B, kind, ts);
+            return cudaMemcpyAsync(dst, src, pitch * B, kind, cst);
         const bool a16 = per % 16 == 0 && (reinterpret_cast<uintptr_t>(dst) & 15) == 0 &&
                          (reinterpret_cast<uintptr_t>(src) & 15) == 0;
         if (a16) {
-            stage_tokens_kernel<<<2 * device_sm_count(), 128, 0, ts>>>(static_cast<uint4*>(dst), static_cast<const uint4*>(src),
+            stage_tokens_kernel<<<2 * device_sm_count(), 128, 0, cst>>>(static_cast<uint4*>(dst), static_cast<const uint4*>(src),
                                                         B, static_cast<long long>(pitch / 16),
                                                         static_cast<long long>(off / 16),
                                                         static_cast<long long>(width / 16));
@@ -791,7 +806,7 @@ int qstate_scan_host(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong,
         cudaError_t err = cudaSuccess;
         for (int bb = 0; bb < B && err == cudaSuccess; ++bb)
             err = cudaMemcpyAsync(static_cast<char*>(dst) + bb * pitch + off,
-                                  static_cast<const char*>(src) + bb * pitch + off, width, kind, ts);
+                                  static_cast<const char*>(src) + bb * pitch + off, width, kind, cst);
         return err;
     };
     qstate_buf* src = ping;
@@ -799,12 +814,12 @@ int qstate_scan_host(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong,
     int in_pong = 0, w = w_index0;
     cudaError_t e = cudaSuccess;
     cudaEvent_t ev_in = nullptr, ev_out = nullptr;
-    // Inputs of chunk c + 1 are queued on the copy stream before the readouts of chunk c, so
-    // they move while chunk c computes (they fill other tokens of the device buffers); the
-    // readouts of chunk c follow once it is done.
+    // Inputs of chunk c + 1 are queued on the copy stream once chunk c's scan is queued, so they
+    // move while chunk c computes (they fill other tokens of the device buffers); the readouts of
+    // chunk c follow on the readout stream once it is done.
     auto stage_inputs = [&](int c0, int c1) {
         for (const Item& it : in)
-            if (it.h && e == cudaSuccess) e = copy_tokens(it.d, it.h, it.per, c0, c1, cudaMemcpyHostToDevice);
+            if (it.h && e == cudaSuccess) e = copy_tokens(it.d, it.h, it.per, c0, c1, cudaMemcpyHostToDevice, ts);
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev_in, cudaEventDisableTiming);
         if (e == cudaSuccess) e = cudaEventRecord(ev_in, ts);
     };
@@ -828,18 +843,20 @@ int qstate_scan_host(const qstate_cfg* cfg, qstate_buf* ping, qstate_buf* pong,
         if (c1 < t_end) stage_inputs(c1, c1 + chunk < t_end ? c1 + chunk : t_end);
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev_out, cudaEventDisableTiming);
         if (e == cudaSuccess) e = cudaEventRecord(ev_out, cs);
-        if (e == cudaSuccess) e = cudaStreamWaitEvent(ts, ev_out, 0);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(rs, ev_out, 0);
         if (ev_out) cudaEventDestroy(ev_out);
         ev_out = nullptr;
-        if (e == cudaSuccess) e = copy_tokens(o_host, o_dev, H * cfg->dv * f4, c0, c1, cudaMemcpyDeviceToHost);
+        if (e == cudaSuccess) e = copy_tokens(o_host, o_dev, H * cfg->dv * f4, c0, c1, cudaMemcpyDeviceToHost, rs);
     }
     if (ev_in) cudaEventDestroy(ev_in);
-    // the compute stream completes only after the last readout copy
-    if (e == cudaSuccess && rc == QSTATE_OK) {
-        e = cudaEventCreateWithFlags(&ev_out, cudaEventDisableTiming);
-        if (e == cudaSuccess) e = cudaEventRecord(ev_out, ts);
-        if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, ev_out, 0);
+    // the compute stream completes only after the last readout copy (also after a failure, so
+    // that no copy on the library's stream is left unordered)
+    {
+        cudaError_t e1 = cudaEventCreateWithFlags(&ev_out, cudaEventDisableTiming);
+        if (e1 == cudaSuccess) e1 = cudaEventRecord(ev_out, rs);
+        if (e1 == cudaSuccess) e1 = cudaStreamWaitEvent(cs, ev_out, 0);
         if (ev_out) cudaEventDestroy(ev_out);
+        if (e == cudaSuccess) e = e1;
     }
     if (rc) return rc;
     if (e != cudaSuccess) return cuda_fail(e, "host staging");
