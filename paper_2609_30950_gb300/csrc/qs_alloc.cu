@@ -155,9 +155,12 @@ __global__ void __launch_bounds__(kThreads, 2) alloc_kernel(const AllocParams p)
     const int gsz = p.group_heads * p.dk;
     const int gshift = (gsz & (gsz - 1)) == 0 ? __ffs(gsz) - 1 : -1;
     const int ngroups = p.unit_row ? N / gsz : 0;
-    float* ms_s = reinterpret_cast<float*>(key + N);                 // EMA statistics
-    float* mr_s = ms_s + N;
-    float* Rs = mr_s + N;                                              // row unit: ranges, a padding
+    // the EMA statistics are read once each, from global memory (the write-back just wrote
+    // them: L2); only the ranges, read twice, are staged
+    const size_t base = static_cast<size_t>(blockIdx.x) * N;
+    const float* ms_s = p.uniform ? nullptr : p.ema_s + base;
+    const float* mr_s = p.uniform ? nullptr : p.ema_r + base;
+    float* Rs = reinterpret_cast<float*>(key + N);                     // row unit: ranges, a padding
                                                                        // word after each group
     float* gmean = Rs + (p.unit_row ? N + ngroups : 0);
     int* hist = reinterpret_cast<int*>(gmean + ((ngroups + 3) & ~3));
@@ -165,18 +168,13 @@ __global__ void __launch_bounds__(kThreads, 2) alloc_kernel(const AllocParams p)
     int* sel = redi + 72;                                              // H*, rank, low prefix
     uint8_t* wv = reinterpret_cast<uint8_t*>(sel + 4);
     const int tid = threadIdx.x;
-    const size_t base = static_cast<size_t>(blockIdx.x) * N;
 
-    // 1. statistics and ranges staged in shared memory (independent coalesced loads); mean R^2
-    //    of each output-normalisation group, summed in row order (row unit).  Group g's ranges
-    //    sit at stride gsz + 1, so the threads summing different groups in lockstep hit
-    //    different banks.
+    // 1. ranges staged in shared memory (row unit; independent coalesced loads); mean R^2 of
+    //    each output-normalisation group, summed in row order.  Group g's ranges sit at stride
+    //    gsz + 1, so the threads summing different groups in lockstep hit different banks.
     if (!p.uniform) {
-        for (int u = tid; u < N; u += kThreads) {
-            ms_s[u] = p.ema_s[base + u];
-            mr_s[u] = p.ema_r[base + u];
-            if (p.unit_row) Rs[u + group_of(u, gsz, gshift)] = p.range[base + u];
-        }
+        if (p.unit_row)
+            for (int u = tid; u < N; u += kThreads) Rs[u + group_of(u, gsz, gshift)] = p.range[base + u];
         __syncthreads();
         if (p.unit_row) {
             // one thread per group, its sum a chain of gsz dependent additions: the next 16
@@ -352,7 +350,7 @@ __global__ void __launch_bounds__(kThreads, 2) alloc_kernel(const AllocParams p)
 
 cudaError_t launch_alloc(const AllocParams& p, cudaStream_t stream) {
     const int ngroups = p.unit_row ? p.units / (p.group_heads * p.dk) : 0;
-    const size_t smem = static_cast<size_t>(p.units) * 4 * 3 + (p.unit_row ? (p.units + ngroups) * 4 : 0) +
+    const size_t smem = static_cast<size_t>(p.units) * 4 + (p.unit_row ? (p.units + ngroups) * 4 : 0) +
                         ((ngroups + 3) & ~3) * 4 + 1024 * 4 + 72 * 4 + 4 * 4 + p.units + 16;
     cudaError_t e = cudaFuncSetAttribute(alloc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
