@@ -135,6 +135,24 @@ __device__ __forceinline__ void cp_async4(void* smem, const void* gmem) {
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
 
+// Decoding in the update layout: a lane's CPL codes of a row of width w (up to 16) at bit
+// lane CPL w, without a branch on the width: three words are read and the lane's bits taken
+// from their 64-bit window, so the decoding of consecutive rows of different
+// widths can overlap.  `row` is followed by >= 12 readable bytes.
+template <int CPL>
+__device__ __forceinline__ void extract_codes_flat(const uint8_t* row, int lane, int w,
+                                                   uint32_t (&u)[CPL]) {
+    const uint32_t* words = reinterpret_cast<const uint32_t*>(row);
+    const int P = lane * CPL * w;
+    const int idx = P >> 5, sh = P & 31;
+    const uint32_t mask = (1u << w) - 1u;
+    const uint32_t lo = __funnelshift_r(words[idx], words[idx + 1], sh);
+    const uint32_t hi = __funnelshift_r(words[idx + 1], words[idx + 2], sh);
+    const uint64_t chunk = (static_cast<uint64_t>(hi) << 32) | lo;
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) u[c] = static_cast<uint32_t>(chunk >> (c * w)) & mask;
+}
+
 // ---- row layout: 32 consecutive codes of one row per lane ---------------------------------------
 // The lane's codes occupy the 4W bytes at byte 4 W q of the row (q = its part), a whole number of
 // words: code c of the run sits at bits [c W, c W + W) of those words.
@@ -505,7 +523,7 @@ __global__ void __launch_bounds__(NW * 32, CHUNK ? 1 : 2) wb_row_kernel(const Wb
             for (int jr = 0; jr < NSL; ++jr) {
                 const int i = warp * RPW + jr * RS + half;
                 uint32_t u[4];
-                extract_codes<4>(pay + sm.off_in[i], cl, static_cast<int>(S.w_in[i]), u);
+                extract_codes_flat<4>(pay + sm.off_in[i], cl, static_cast<int>(S.w_in[i]), u);
                 const float4 as = sm.deqAS[i];
                 const float2 A2 = make_float2(as.x, as.y), S2 = make_float2(as.z, as.w), B2 = sm.deqB[i];
 #pragma unroll
@@ -526,7 +544,7 @@ __global__ void __launch_bounds__(NW * 32, CHUNK ? 1 : 2) wb_row_kernel(const Wb
             for (int rr = 0; rr < 4; ++rr) {
                 const int r = r4 + rr;
                 uint32_t u[CPL];
-                extract_codes<CPL>(pay + offs[rr], lane, static_cast<int>((w4 >> (8 * rr)) & 0xFFu), u);
+                extract_codes_flat<CPL>(pay + offs[rr], lane, static_cast<int>((w4 >> (8 * rr)) & 0xFFu), u);
                 const float4 as = sm.deqAS[i0 + rr];
                 const float2 A2 = make_float2(as.x, as.y), S2 = make_float2(as.z, as.w), B2 = sm.deqB[i0 + rr];
 #pragma unroll
