@@ -97,3 +97,51 @@ def test_scan_partition_setter_checks_its_range(lib):
     assert lib.qstate_set_scan_partitions(-1) == QSTATE_EINVAL
     for n in (8, 1, 0):
         assert lib.qstate_set_scan_partitions(n) == QSTATE_OK
+
+
+def _part_count(lib, w, parts, form=0, s_code=False, beta=True):
+    """qstate_scan_partition_count on host-only arguments: placeholder device addresses (the
+    call only checks them for NULL and never dereferences them)."""
+    import paper_2609_30950_gb300 as q
+    cfg = q.Config.from_workload(w, interval_form=form).c()
+    A = 1 << 20
+    x = q._Inputs(A, A, A, None if s_code else A, A if s_code else None, A if s_code else None,
+                  A if beta else None, w.T, None, None)
+    st = q._Stats(A, A, A)
+    assert lib.qstate_set_scan_partitions(parts) == 0
+    try:
+        return lib.qstate_scan_partition_count(ct.byref(cfg), ct.byref(x), ct.byref(st))
+    finally:
+        lib.qstate_set_scan_partitions(0)
+
+
+def test_scan_partition_count_rule(lib):
+    """Batch partitions of a scan: 4 in the token form and 2 in the chunked form by default, at
+    most one per batch element, and fewer where a partition would start off a 16-byte boundary
+    in any array."""
+    import synth
+    kda = synth.scaled(synth.WORKLOADS["kda_decode"], B=16, H=8, T=48)
+    assert _part_count(lib, kda, 0, s_code=True) == 4
+    assert _part_count(lib, kda, 0, form=1) == 2
+    assert _part_count(lib, kda, 8) == 8
+    assert _part_count(lib, synth.scaled(kda, B=3), 8) == 3
+    assert _part_count(lib, synth.scaled(kda, B=1), 0) == 1
+    assert _part_count(lib, kda, 1) == 1
+    # head unit with H = 3: 3 width bytes per batch element, so a partition may start only at a
+    # multiple of 16 elements; with B = 32 that leaves the split at element 16
+    gdn = synth.scaled(synth.WORKLOADS["gdn_decode"], B=32, H=3, T=16)
+    assert _part_count(lib, gdn, 4) == 2
+    assert _part_count(lib, gdn, 8) == 2
+    # per-head rates of an odd token count: 4 T H bytes per element, T H = 3 x 17
+    gdn_odd = synth.scaled(synth.WORKLOADS["gdn_decode"], B=4, H=16, T=17)
+    assert _part_count(lib, gdn_odd, 4) == 4          # 4 x 17 x 16 = 1088: aligned
+    kda_odd = synth.scaled(kda, B=4, T=17)            # rate codes: T H dk bytes, aligned
+    assert _part_count(lib, kda_odd, 4, s_code=True) == 4
+    # an invalid configuration or missing statistics: 0
+    import paper_2609_30950_gb300 as q
+    cfg = q.Config.from_workload(kda).c()
+    x = q._Inputs(1 << 20, 1 << 20, 1 << 20, 1 << 20, None, None, 1 << 20, kda.T, None, None)
+    assert lib.qstate_scan_partition_count(ct.byref(cfg), ct.byref(x), None) == 0
+    bad = q.Config.from_workload(kda, C=0).c()
+    st = q._Stats(1 << 20, 1 << 20, 1 << 20)
+    assert lib.qstate_scan_partition_count(ct.byref(bad), ct.byref(x), ct.byref(st)) == 0
