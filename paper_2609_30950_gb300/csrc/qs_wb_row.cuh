@@ -855,11 +855,17 @@ __global__ void __launch_bounds__(NW * 32, CHUNK ? 1 : 2) wb_row_kernel(const Wb
                 const float2* crow = sm.rc.cand[warp][lane / TPR];
                 float bsse = INFINITY;
                 int bk = kNFit - 1;
+                // each round's two candidates are loaded one round ahead
+                float2 pA = crow[kNFit - 1], pB = crow[kNFit - 2];
 #pragma unroll 1
                 for (int k = kNFit - 1; k >= 0; k -= 2) {
                     // candidates k and k - 1 in one round (k - 1 may not exist)
                     const bool two = k >= 1;
-                    const float2 cA = crow[k], cB = crow[two ? k - 1 : k];
+                    const float2 cA = pA, cB = two ? pB : pA;
+                    if (k >= 3) {
+                        pA = crow[k - 2];
+                        pB = crow[k - 3];
+                    }
                     const float LA = -nf * cA.y, LB = -nf * cB.y;
                     float lbA = 0.0f;
 #pragma unroll
