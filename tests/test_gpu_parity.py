@@ -223,14 +223,16 @@ def test_fp32_recurrence_free_running(qs, orc, name):
 
 # --------------------------------------------------------------- quantised write-backs, lockstep
 def _lockstep(qs, orc, w, fit_every=1, log_decay=False, sample_b=None, max_wb=None, weight_kind=0,
-              interval_form=0, inputs=None):
+              interval_form=0, inputs=None, oracle_parallel=False):
     """Run the oracle free; before every write-back copy its state into the GPU, run one
     qstate_step and compare the GPU's write-back with the oracle's.  With sample_b, the GPU
     runs the full batch and only those batch elements are injected and compared (the oracle
     runs a B=1 configuration per sampled element, one host thread each).  interval_form
     selects the library's token-by-token or chunked computation of each interval (the oracle
     is always token by token).  Returns the per-write-back report and the oracle's
-    free-running readouts per compared element."""
+    free-running readouts per compared element.  oracle_parallel runs the oracle's OpenMP
+    build (the heads of a write-back on several threads; the same results bit for bit, pinned
+    on the CPU)."""
     cfgq = qs.Config.from_workload(w, fit_every=fit_every, weight_kind=weight_kind,
                                    interval_form=interval_form)
     cfgo_full = orc.Cfg.from_workload(w, fit_every=fit_every, weight_kind=weight_kind)
@@ -289,7 +291,7 @@ def _lockstep(qs, orc, w, fit_every=1, log_decay=False, sample_b=None, max_wb=No
         def orc_step(key):
             S = states[key]
             return orc.step(cfgo, S["src"], S["dst"], orc_inp[key], t0, t1, wi, S["o"], S["ms"], S["mr"],
-                            S["R"], orc_code[key], s_lut, want_x=True)
+                            S["R"], orc_code[key], s_lut, want_x=True, parallel=oracle_parallel)
         if len(states) > 1:
             xos = dict(zip(states, pool.map(orc_step, list(states))))
         else:
